@@ -1,0 +1,423 @@
+#!/usr/bin/env python
+"""Benchmark of the RPS scoring path (rps_score_step / rps_select_pivots /
+rps_score_branches / rps_commit) on GB300.
+
+A step is one pass of the whole path over one decoding step's synthetic logits:
+row statistics of the masked base rows (top-k mode), standard commit and pivot
+selection, row statistics of the lookahead rows, benefit scores and the commit
+decision. The headline workload is one generation step: 256 masked positions,
+vocab 126,464, bf16 logits, 1 base + 8 lookahead branches (4 pivots x top-2).
+
+Timing: the five launches of a step are captured in one CUDA graph; each timed
+replay is preceded by a 256 MB write that flushes L2 and bracketed by CUDA
+events on the launching stream; event nodes inside the graph time the lookahead
+row-statistics kernel (the dominant kernel) on the same stream. SM clocks and
+throttle reasons are sampled with nvidia-smi during the timed region.
+
+`value` is scored logit rows per second over the whole job (N replicas, one per
+GPU, no collective in the data path: weak scaling). `e2e` is the same metric
+through the C ABI with the step's logits in pinned host memory: host-to-device
+copy, the step, and the read-back of the decisions are all inside the timed
+region. `--impl reference` times the CPU oracle (the only other implementation
+of this path) on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = "lookahead-scoring logit rows/s and achieved HBM GB/s (fraction of GB300 peak)"
+HEADLINE = "step"
+OTHERS = ("step-50", "step-10", "long", "block", "serve")
+FLUSH_BYTES = 256 << 20
+FALLBACK_HBM_GBS = 6800.0
+
+
+def describe(w) -> str:
+    return (f"{w.name}: {w.n_req} request(s) x {w.L} positions, vocab {w.V}, {w.dtype} logits, "
+            f"1 base + {w.n_branch} lookahead branches ({w.n_pivots} pivots x top-{w.tokens_per_pivot}), "
+            f"mixture {w.mixture}, masked {'ragged ' + str(w.ragged) if w.ragged else w.masked_frac}")
+
+
+def peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = [l.split(",") for l in open(self.path).read().splitlines() if l.strip()]
+        os.unlink(self.path)
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+                for n, v in zip(names, r[5:9]):
+                    if v.strip().lower() == "active":
+                        reasons.add(n)
+            except (ValueError, IndexError):
+                continue
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+class Workload:
+    """Device-resident inputs, buffers and the captured step of one workload."""
+
+    def __init__(self, w, prm, device):
+        import torch
+        from paper_2608_11742_gb300 import rps, synth
+        self.w, self.prm, self.device = w, prm, device
+        dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+        self.logits = torch.empty((w.n_req, 1 + w.n_branch, w.L, w.V), dtype=dt, device=device)
+        valid = w.valid_rows()
+        synth.device_fill(self.logits, w.seed, w.mixture,
+                          valid=None if valid is None else torch.from_numpy(valid).to(device))
+        mpos, mcnt = w.mask()
+        self.mpos = torch.from_numpy(mpos).to(device)
+        self.mcnt = torch.from_numpy(mcnt).to(device)
+        self.step = rps.Step(w.n_req, w.L, w.V, prm, device)
+        self.stream = torch.cuda.Stream(device)
+        self.ev = None
+        with torch.cuda.stream(self.stream):
+            self.step.run(self.logits, self.mpos, self.mcnt)
+        self.stream.synchronize()
+        status, detail = rps.rps_poll_device_status()
+        if status != rps.RPS_OK:
+            raise RuntimeError(f"device error bits {detail:#x}")
+        self.base_rows = int(mcnt.sum())
+        self.branch_rows = int(self.step.piv.n_branch_rows.sum())
+        self.graph = self._capture()
+
+    def _capture(self):
+        import torch
+        g = torch.cuda.CUDAGraph()
+        try:
+            ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+        except TypeError:  # torch without external events: time the kernel in its own graph
+            ev = None
+        with torch.cuda.graph(g, stream=self.stream):
+            self.step.score_base(self.logits, self.mpos, self.mcnt)
+            self.step.select(self.mpos, self.mcnt)
+            if ev:
+                ev[0].record()
+            self.step.score_branch_rows(self.logits)
+            if ev:
+                ev[1].record()
+            self.step.score(self.logits)
+            self.step.decide()
+        self.ev = ev
+        if ev is None:
+            self.k1_graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(self.k1_graph, stream=self.stream):
+                self.step.score_branch_rows(self.logits)
+        return g
+
+    def rows(self):
+        return self.base_rows + self.branch_rows
+
+    def bytes(self):
+        return self.rows() * self.w.V * self.w.elem_bytes
+
+    def branch_bytes(self):
+        return self.branch_rows * self.w.V * self.w.elem_bytes
+
+    def time(self, steps, warmup, flush):
+        import torch
+        s = self.stream
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        step_ms, k1_ms = [], []
+        for i in range(warmup + steps):
+            with torch.cuda.stream(s):
+                flush.add_(1)
+                e0.record(s)
+                self.graph.replay()
+                e1.record(s)
+            s.synchronize()
+            if i >= warmup:
+                step_ms.append(e0.elapsed_time(e1))
+                if self.ev:
+                    k1_ms.append(self.ev[0].elapsed_time(self.ev[1]))
+        if not self.ev:
+            for i in range(warmup + steps):
+                with torch.cuda.stream(s):
+                    flush.add_(1)
+                    e0.record(s)
+                    self.k1_graph.replay()
+                    e1.record(s)
+                s.synchronize()
+                if i >= warmup:
+                    k1_ms.append(e0.elapsed_time(e1))
+        return step_ms, k1_ms
+
+    def e2e(self, steps, warmup):
+        """Same step through the C ABI from pinned host buffers, copies included."""
+        import torch
+        host = torch.empty(self.logits.shape, dtype=self.logits.dtype, pin_memory=True)
+        host.copy_(self.logits)
+        hpos = self.mpos.cpu().pin_memory()
+        hcnt = self.mcnt.cpu().pin_memory()
+        c = self.step.commit
+        outs = [c.winner, c.commit_pos, c.commit_tok, c.mask_cnt, c.mask_pos, self.step.piv.n_commit,
+                self.step.piv.commit_pos, self.step.piv.commit_tok]
+        hout = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+        dlog, dpos, dcnt = torch.empty_like(self.logits), torch.empty_like(self.mpos), torch.empty_like(self.mcnt)
+        s = self.stream
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ms = []
+        for i in range(warmup + steps):
+            with torch.cuda.stream(s):
+                e0.record(s)
+                dlog.copy_(host, non_blocking=True)
+                dpos.copy_(hpos, non_blocking=True)
+                dcnt.copy_(hcnt, non_blocking=True)
+                self.step.run(dlog, dpos, dcnt)
+                for h, d in zip(hout, outs):
+                    h.copy_(d, non_blocking=True)
+                e1.record(s)
+            s.synchronize()
+            if i >= warmup:
+                ms.append(e0.elapsed_time(e1))
+        h2d = host.numel() * host.element_size() + hpos.numel() * 4 + hcnt.numel() * 4
+        d2h = sum(h.numel() * h.element_size() for h in hout)
+        del dlog
+        return ms, h2d, d2h
+
+
+def cpu_sample(w, n_take: int = 64):
+    """A bounded sample of one step's rows, in the step's proportions: base rows
+    (scored in top-k mode) and lookahead rows (statistics only)."""
+    import numpy as np
+    from paper_2608_11742_gb300 import synth
+    mpos, mcnt = w.mask()
+    rng = np.random.default_rng(0)
+    n_base = max(1, int(round(n_take / (1 + w.n_branch))))
+    base, branch = [], []
+    for i in range(n_take):
+        q = int(rng.integers(0, w.n_req))
+        pos = int(mpos[q, int(rng.integers(0, max(int(mcnt[q]), 1)))])
+        b = 0 if i < n_base else int(rng.integers(1, 1 + w.n_branch))
+        (base if b == 0 else branch).append(synth.row_logits(w.seed, w.V, q, b, pos, w.mixture, w.dtype))
+    return np.stack(base), np.stack(branch)
+
+
+def time_oracle(sample, k_max: int, budget_s: float):
+    """Rows per second of the oracle as it stands (single thread) over the sample, repeated for budget_s."""
+    from oracle import default as oracle_default
+    o = oracle_default()
+    rb, rr = sample
+    done, t0, elapsed = 0, time.perf_counter(), 0.0
+    while elapsed < budget_s:
+        o.row_stats(rb, k_max)
+        o.row_stats(rr, 0)
+        done += len(rb) + len(rr)
+        elapsed = time.perf_counter() - t0
+    return done / elapsed, done, elapsed
+
+
+def cpu_baseline(w, prm, budget_s: float):
+    sample = cpu_sample(w)
+    rows_s, done, elapsed = time_oracle(sample, prm.k_max, budget_s)
+    return {"value": rows_s, "unit": "rows/s", "cores": 1, "kind": "oracle",
+            "sample": f"{done} rows of the {w.name} workload ({len(sample[0])} base rows in top-k mode and "
+                      f"{len(sample[1])} lookahead rows, repeated) scored by the single-threaded fp64 oracle in "
+                      f"{elapsed:.1f} s ({rows_s * w.V * w.elem_bytes / 1e9:.3f} GB/s)"}
+
+
+def run_gpu(args):
+    import torch
+    from paper_2608_11742_gb300 import configs, rps
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    flush = torch.zeros(FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    peak, peak_kind = peaks()
+
+    w = configs.ALL[args.workload]
+    prm = w.params(configs.EXERCISE)
+    wl = Workload(w, prm, device)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        step_ms, k1_ms = wl.time(args.steps, args.warmup, flush)
+    clocks = clk.summary()
+    t_step = statistics.mean(step_ms)
+    if world > 1:
+        t = torch.tensor([t_step], device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        t_step = float(t.item())
+    rows = wl.rows()
+    value = world * rows / (t_step / 1e3)
+    k1 = statistics.mean(k1_ms)
+    achieved = wl.branch_bytes() / (k1 / 1e3) / 1e9
+    traffic = None
+    tf = ROOT / "profiles" / "traffic.json"
+    if tf.exists():
+        d = json.loads(tf.read_text())
+        traffic = d.get(args.workload)
+
+    out = {
+        "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": describe(w), "input_dtype": w.dtype,
+                   "params": {"k_max": prm.k_max, "r": prm.r, "tau_pivot": prm.tau_pivot, "tau": prm.tau,
+                              "lambda": prm.lam, "n_pivots": prm.n_pivots, "tokens_per_pivot": prm.tokens_per_pivot},
+                   "rows_per_step": rows, "base_rows": wl.base_rows, "lookahead_rows": wl.branch_rows,
+                   "bytes_per_step": wl.bytes(), "l2": "flushed (256 MB write) before every timed step",
+                   "parallelism": f"{world} independent replica(s), no collective"},
+        "achieved_gbs": wl.bytes() / (t_step / 1e3) / 1e9,
+        "frac_of_hbm_peak": wl.bytes() / (t_step / 1e3) / 1e9 / peak,
+        "roofline": {"bound": "hbm", "kernel": "row statistics of the lookahead rows (statistics-only mode)",
+                     "achieved": achieved, "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "algorithmic_bytes_per_launch": wl.branch_bytes(), "launch_ms": k1},
+        "clocks": clocks,
+        "gpu_launches": rps.Step.LAUNCHES * args.steps,
+    }
+    del wl
+    torch.cuda.empty_cache()
+
+    if not args.skip_others:
+        others = {}
+        for name in OTHERS:
+            wo = configs.ALL[name]
+            x = Workload(wo, wo.params(configs.EXERCISE), device)
+            sm, km = x.time(max(5, args.steps // 2), 3, flush)
+            ts = statistics.mean(sm)
+            kk = statistics.mean(km)
+            others[name] = {"rows_per_step": x.rows(), "step_us": ts * 1e3, "p50_step_us": statistics.median(sm) * 1e3,
+                            "p90_step_us": sorted(sm)[int(0.9 * (len(sm) - 1))] * 1e3,
+                            "rows_per_s": x.rows() / (ts / 1e3), "gbs": x.bytes() / (ts / 1e3) / 1e9,
+                            "frac": x.bytes() / (ts / 1e3) / 1e9 / peak,
+                            "lookahead_kernel_gbs": x.branch_bytes() / (kk / 1e3) / 1e9}
+            del x
+            torch.cuda.empty_cache()
+        out["other_workloads"] = others
+
+    if not args.skip_e2e:
+        wl = Workload(w, prm, device)
+        ms, h2d, d2h = wl.e2e(max(3, args.steps // 4), 2)
+        te = statistics.mean(ms)
+        out["e2e"] = {"value": world * rows / (te / 1e3), "unit": "rows/s", "h2d_bytes_per_step": h2d,
+                      "d2h_bytes_per_step": d2h, "ms_per_step": te}
+        del wl
+        torch.cuda.empty_cache()
+
+    if rank == 0 and world == 1 and not args.skip_cpu:
+        out["cpu_baseline"] = cpu_baseline(w, prm, args.cpu_seconds)
+        out["cpu_baseline"].pop("seconds", None)
+
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out))
+
+
+def run_reference(args):
+    """The CPU oracle as the reference arm, on the host cores, same metric and workload."""
+    from paper_2608_11742_gb300 import configs
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    w = configs.ALL[args.workload]
+    prm = w.params(configs.EXERCISE)
+    per_step = max(0.5, args.cpu_seconds / max(1, args.steps + args.warmup))
+    sample = cpu_sample(w)
+    vals = []
+    for i in range(args.warmup + args.steps):
+        rows_s, _, _ = time_oracle(sample, prm.k_max, per_step)
+        if i >= args.warmup:
+            vals.append(rows_s)
+    value = statistics.mean(vals)
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": None, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": describe(w), "input_dtype": w.dtype},
+           "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                            "sample": f"each step: about {per_step:.1f} s of the single-threaded fp64 oracle on a "
+                                      f"64-row sample of the workload ({len(sample[0])} base rows in top-k mode, "
+                                      f"{len(sample[1])} lookahead rows)"},
+           "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", default=HEADLINE)
+    ap.add_argument("--skip-others", action="store_true")
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-cpu", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

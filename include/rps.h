@@ -1,0 +1,273 @@
+/*
+ * rps.h -- C ABI of the GB300 scoring path of Ripple-Pivot Search (RPS).
+ *
+ * One decoding step of RPS (Algorithm 1 of the paper) on logits already in
+ * device memory:
+ *
+ *   rps_score_step      per-row statistics of the masked rows: entropy H(p_i),
+ *                       confidence P_i^max, argmax (Eq. 1), top-k_max support
+ *                       T_i, retained mass mu_i and truncated entropy (Eq. 3)
+ *   rps_select_pivots   confidence-aware standard commit S (Eq. 2, with the
+ *                       fallback of Algorithm 1), remaining set M' = M \ S,
+ *                       pivot selection (Eq. 3), adaptive candidate tokens
+ *                       (Sec. 3.1) and the list of lookahead rows to score
+ *   rps_score_step      again, on the lookahead branches' rows
+ *   rps_score_branches  downstream-benefit score of every candidate (Eq. 4),
+ *                       with the eligible-commit count N_tau (Proposition 1)
+ *   rps_commit          commit-or-abstain decision (Eq. 4 argmax over C
+ *                       including [MASK]; Algorithm 1) and the mask after the step
+ *
+ * Conventions
+ *   - Every array pointer is a caller-owned DEVICE pointer unless stated.
+ *     The library never allocates device memory; per-call scratch comes from a
+ *     caller-owned workspace sized by rps_workspace_bytes.
+ *   - Calls are asynchronous on the given stream (NULL = legacy default stream)
+ *     and return as soon as the work is enqueued.
+ *   - Host-detectable errors (NULL pointers, out-of-range sizes or parameters,
+ *     misaligned logits) return an error status before anything is enqueued and
+ *     write nothing.
+ *   - Bad DATA found by a kernel (a row descriptor outside the logit tensor, a
+ *     mask count above capacity, a row without a finite logit) does not trap:
+ *     the kernel skips the offending item, writes NaN / -1 where it stands, and
+ *     ORs a bit into a sticky per-device error word that rps_poll_device_status
+ *     reads and clears.
+ *   - Results are deterministic for a given input and launch configuration.
+ *   - Layout per request q of n_req, with L positions of capacity:
+ *       mask / base statistics      [q * L + k], k = index in q's mask list
+ *       pivot slot j of P           [q * P + j]
+ *       candidate c of K            [(q * P + j) * K + c]
+ *       lookahead branch b          b = j * K + c of NB = P * K; it is branch
+ *                                   1 + b of the logit tensor (branch 0 = base)
+ *       branch scores               [(q * P + j) * (K + 1) + c], c == K is [MASK]
+ */
+#ifndef RPS_H
+#define RPS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *rps_stream_t;
+
+typedef enum {
+    RPS_OK = 0,
+    RPS_ERR_INVALID_ARG = 1, /* rejected on the host; nothing was enqueued */
+    RPS_ERR_UNSUPPORTED = 2, /* well-formed request outside this build's limits */
+    RPS_ERR_CUDA = 3,        /* a CUDA runtime call (launch, attribute query) failed */
+    RPS_ERR_DEVICE = 4,      /* a kernel flagged bad data; see rps_poll_device_status */
+    RPS_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up (no kernel here waits) */
+} rps_status;
+
+/* Bits of the device error word. */
+#define RPS_DEVERR_ROW_INDEX 0x1u  /* row descriptor outside the logit tensor */
+#define RPS_DEVERR_NONFINITE 0x2u  /* a scored row holds NaN or no finite logit */
+#define RPS_DEVERR_MASK 0x4u       /* mask count above capacity or position out of range */
+#define RPS_DEVERR_TOKEN 0x8u      /* candidate token outside the vocabulary */
+
+typedef enum { RPS_F32 = 0, RPS_BF16 = 1 } rps_dtype;
+
+/* Per-request state after rps_select_pivots. */
+typedef enum {
+    RPS_STATE_SEARCH = 0,       /* lookahead branches are scored this step */
+    RPS_STATE_DONE = 1,         /* M' is empty after the standard commit (Algorithm 1 break) */
+    RPS_STATE_NO_FEASIBLE = 2,  /* no row has mu_i >= tau_pivot: skip the search (Eq. 3) */
+    RPS_STATE_NO_CANDIDATES = 3 /* no pivot has two candidates: skip (|C \ MASK| <= 1) */
+} rps_state;
+
+/* Winner codes written by rps_commit (>= 0 is the committed branch b). */
+#define RPS_WIN_ANCHOR (-1) /* every searched pivot keeps [MASK]: reuse the anchor's logits */
+#define RPS_WIN_SKIP (-2)   /* search skipped: the next step needs a fresh forward pass */
+#define RPS_WIN_DONE (-3)   /* nothing left to decode in this block */
+
+/* Limits of this build. */
+#define RPS_MAX_K 32        /* k_max */
+#define RPS_MAX_PIVOTS 16   /* P */
+#define RPS_MAX_POS 4096    /* L */
+#define RPS_MAX_SEGMENTS 1024
+
+/* Hyper-parameters (Sec. 4 "Implementation details": k_max = 10, r = 0.1,
+ * tau_pivot = 0.9 / 0.95, lambda in [0.1, 0.5]; Appendix C: tau = 0.9). */
+typedef struct {
+    int32_t k_max;            /* |T_i| of Eq. 3, 1..RPS_MAX_K */
+    float r;                  /* reachability ratio of the candidate set, (0, 1] */
+    float tau_pivot;          /* probability-mass constraint of Eq. 3 */
+    float tau;                /* confidence threshold of Eq. 2 (and of N_tau) */
+    float lambda;             /* plausibility weight of Eq. 4, >= 0 */
+    int32_t n_pivots;         /* P: pivot slots scored side by side, 1..RPS_MAX_PIVOTS */
+    int32_t tokens_per_pivot; /* K: candidate tokens per pivot, 1..k_max */
+} rps_params;
+
+/* A logit tensor [n_req][n_branch][n_pos][vocab] in device memory. The vocab
+ * dimension is contiguous; the other strides are in elements. `data` must be
+ * 16-byte aligned and every stride a multiple of 16 bytes, so that each row
+ * starts on a 16-byte boundary; vocab itself is unrestricted. */
+typedef struct {
+    const void *data;
+    int32_t dtype; /* rps_dtype */
+    int32_t n_req, n_branch, n_pos;
+    int64_t vocab;
+    int64_t req_stride, branch_stride, pos_stride;
+} rps_logits;
+
+/* Rows to score, grouped in n_seg segments of capacity cap. Entry i of segment s
+ * is rows[(s * cap + i) * 3 + {0,1,2}] = (req, branch, pos) and its statistics go
+ * to slot s * cap + i of the output arrays. Only i < seg_cnt[s] is read
+ * (seg_cnt is a device array, or NULL for "all cap entries"); pos < 0 marks an
+ * entry to skip (its slot is not written).
+ * Mask form: with rows == NULL, entry i of segment s is
+ * (s, mask_branch, mask_pos[s * cap + i]), so a request's masked rows (seg_cnt =
+ * mask_cnt, cap = L) are scored without building a descriptor list. */
+typedef struct {
+    const int32_t *rows;
+    const int32_t *seg_cnt;
+    int32_t n_seg;
+    int32_t cap;
+    const int32_t *mask_pos;
+    int32_t mask_branch;
+} rps_row_list;
+
+/* Per-row statistics, structure of arrays, one entry per slot. zmax is the
+ * largest logit, lse = log sum_v exp(z_v), pmax = exp(zmax - lse). topk_idx /
+ * topk_logit hold T_i in rank order (logit descending, then token id
+ * ascending), k_max entries per slot; topk_idx == NULL selects the
+ * statistics-only mode (mu, htrunc, topk_* untouched). */
+typedef struct {
+    float *zmax, *lse, *H, *pmax;
+    int32_t *argmax;
+    float *mu, *htrunc;
+    int32_t *topk_idx;
+    float *topk_logit;
+} rps_row_stats;
+
+/* Outputs of rps_select_pivots (all device arrays). */
+typedef struct {
+    int32_t *n_commit;      /* [n_req] |S| */
+    int32_t *commit_pos;    /* [n_req][L] positions of S in mask order */
+    int32_t *commit_tok;    /* [n_req][L] their greedy tokens (Eq. 1) */
+    int32_t *rem_cnt;       /* [n_req] |M'| */
+    int32_t *rem_k;         /* [n_req][L] mask-list index of each M' entry */
+    int32_t *rem_pos;       /* [n_req][L] position of each M' entry */
+    int32_t *state;         /* [n_req] rps_state */
+    int32_t *pivot_k;       /* [n_req][P] mask-list index of pivot j, -1 if empty */
+    int32_t *pivot_pos;     /* [n_req][P] position of pivot j, -1 if empty */
+    int32_t *n_cand;        /* [n_req][P] candidate tokens of pivot j */
+    int32_t *cand_tok;      /* [n_req][P][K] candidate tokens in rank order, -1 padded */
+    uint8_t *branch_valid;  /* [n_req][NB] 1 when branch b is scored */
+    int32_t *branch_off;    /* [n_req][NB] first entry of branch b in its request's list */
+    int32_t *branch_cnt;    /* [n_req][NB] entries of branch b (|M'| - 1 when valid) */
+    int32_t *n_branch_rows; /* [n_req] entries in the request's list */
+    int32_t *branch_rows;   /* [n_req][NB * L][3] (q, 1 + b, pos): an rps_row_list with
+                               n_seg = n_req, cap = NB * L, seg_cnt = n_branch_rows */
+} rps_pivots;
+
+/* Outputs of rps_score_branches, [n_req][P][K + 1] each (slot K is [MASK]);
+ * slots that are not scored hold NaN and n_tau = -1. */
+typedef struct {
+    float *mean_H;  /* mean downstream entropy H-bar_c */
+    int32_t *n_tau; /* N_tau(c) of Proposition 1 */
+    float *log_a;   /* log p_anchor(c), log P_anchor^max for [MASK] */
+    float *score;   /* Eq. 4 */
+} rps_branch_scores;
+
+/* Outputs of rps_commit. */
+typedef struct {
+    int32_t *best_slot; /* [n_req][P] argmax slot of each searched pivot (K = [MASK]) */
+    float *gain;        /* [n_req][P] score(best) - score([MASK]) */
+    int32_t *winner;    /* [n_req] branch b, or RPS_WIN_ANCHOR / _SKIP / _DONE */
+    int32_t *commit_pos, *commit_tok; /* [n_req] committed pivot and token, -1 if none */
+    float *margin;      /* [n_req] gain of the committed pivot, 0 if none */
+    int32_t *mask_pos;  /* [n_req][L] mask after the step (M' minus the committed pivot) */
+    int32_t *mask_cnt;  /* [n_req] */
+} rps_commit_out;
+
+/* Bytes of workspace rps_score_step needs for up to max_rows row slots
+ * (n_seg * cap) of `vocab` logits with top-k size k_max (0 for statistics
+ * only). Returns 0 for invalid arguments. */
+size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t k_max);
+
+/* Zero a workspace (asynchronously on `stream`). A workspace must be zeroed
+ * once before its first use; every completed rps_score_step leaves it ready
+ * for the next call. One workspace must not serve two calls that can overlap. */
+rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream);
+
+/*
+ * Row statistics (Sec. 2 notation; Eq. 1; Eq. 3) of every listed row:
+ * zmax, lse, H = -sum_v p_v log p_v, pmax = P^max, argmax (lowest token on
+ * ties), and in top-k mode T_i (k_max tokens by logit desc / token asc),
+ * mu = sum_{T_i} p_v and htrunc = -sum_{T_i} p_v log p_v (not renormalised).
+ * fp32 arithmetic; argmax and T_i are exact (taken on the input values).
+ * Errors: RPS_ERR_INVALID_ARG for NULL pointers, a misaligned tensor, sizes out
+ * of range or a workspace smaller than rps_workspace_bytes(n_seg * cap, vocab,
+ * k); RPS_ERR_UNSUPPORTED above RPS_MAX_K / RPS_MAX_SEGMENTS.
+ */
+rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                          const rps_row_stats *out, void *d_ws, size_t ws_bytes, rps_stream_t stream);
+
+/*
+ * Standard commit and pivot selection for n_req requests (Eq. 2, Eq. 3,
+ * Sec. 3.1, Algorithm 1). `base` holds top-k-mode statistics of each request's
+ * masked rows in mask order ([q * L + k], k < mask_cnt[q]); mask_pos lists
+ * distinct positions. Per request:
+ *   S = {i in M : pmax_i >= tau}, or the single most confident row (lowest
+ *   position on ties) when that is empty; S is committed to argmax tokens.
+ *   M' = M \ S. Feasible rows: mu_i >= tau_pivot. Pivots: up to P feasible
+ *   rows by truncated entropy (descending, lower position on ties).
+ *   Candidates: tokens of T_{i*} with z_v - zmax >= log r (that is
+ *   p(v) >= r P^max), in rank order, at most K; a pivot is searched when it has
+ *   at least two. Branch b = j * K + c lists M' without pivot j.
+ * Errors: RPS_ERR_INVALID_ARG for NULL pointers or sizes out of range;
+ * RPS_ERR_UNSUPPORTED when L > RPS_MAX_POS or P > RPS_MAX_PIVOTS.
+ */
+rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
+                             const int32_t *d_mask_cnt, const rps_params *prm, const rps_pivots *out,
+                             rps_stream_t stream);
+
+/*
+ * Downstream-benefit scores (Eq. 4; N_tau of Proposition 1). For searched pivot
+ * j with D_j = M' \ {i*_j} and n = |M'| - 1:
+ *   mean_H = (1/n) sum_{i in D_j} H(p_i^c)  (0 when n == 0)
+ *   n_tau  = #{i in D_j : pmax_i^c >= tau}
+ *   log_a  = z_anchor(i*_j, c) - lse_anchor(i*_j); for [MASK] zmax - lse
+ *   score  = -mean_H + lambda * log_a  (the plausibility term is dropped when
+ *            lambda == 0)
+ * Token candidates read `branch` (statistics-only mode is enough) in the
+ * compact layout of piv->branch_rows; [MASK] reads the anchor statistics of
+ * the rows of D_j ([q * L + k], like `base`). The anchor's pivot-row logits are
+ * read from branch `anchor_branch` of `anchor_logits`.
+ */
+rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_branch,
+                              const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req,
+                              int32_t L, const rps_pivots *piv, const rps_params *prm,
+                              const rps_branch_scores *out, rps_stream_t stream);
+
+/*
+ * Commit decision (Algorithm 1; Eq. 4). Per searched pivot j the best slot is
+ * the argmax of score over its valid tokens and [MASK]; ties keep [MASK], then
+ * the higher-ranked token. gain_j = score(best) - score([MASK]). The request
+ * commits the pivot with the largest gain_j > 0 (lower position on ties) to
+ * its best token, or abstains. out->mask_* receives M' minus the committed
+ * pivot and may alias the mask arrays given to rps_select_pivots.
+ */
+rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
+                      const rps_params *prm, const rps_commit_out *out, rps_stream_t stream);
+
+/* Synchronise `stream`, then read and clear the calling device's error word.
+ * Returns RPS_OK or RPS_ERR_DEVICE (with the RPS_DEVERR_* bits in *detail when
+ * detail != NULL), or RPS_ERR_CUDA if the synchronisation itself failed. */
+rps_status rps_poll_device_status(rps_stream_t stream, uint32_t *detail);
+
+/* Static description of a status code. */
+const char *rps_status_string(rps_status status);
+
+/* ABI version, major * 10000 + minor * 100 + patch. */
+int32_t rps_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RPS_H */

@@ -39,11 +39,15 @@ class Params:
 
 # Paper defaults (LLaDA) with the four-pivot, top-2 layout of the workloads.
 PAPER = Params()
-# Setting under which every masked row is feasible, so pivots, lookahead branches,
-# commits and abstentions all occur on the synthetic logits (with tau_pivot = 0.9
-# no synthetic row at vocab 126,464 reaches the mass constraint and every step
-# takes the skip path of Algorithm 1).
-EXERCISE = Params(tau_pivot=0.0)
+# Setting under which every stage of the step runs on the synthetic logits. With
+# the paper's tau_pivot = 0.9 no synthetic row at vocab 126,464 reaches the mass
+# constraint and every step takes the skip path of Algorithm 1. With every row
+# feasible but tau = 0.9, the truncated-entropy argmax lands on the one-spike
+# rows, whose second token is ~8 nats down (a single candidate: skip again).
+# tau = 0.05 commits those rows in the standard commit, so the pivots come from
+# the flatter rows, which have several candidates, and the lookahead branches are
+# scored every step.
+EXERCISE = Params(tau=0.05, tau_pivot=0.0)
 
 
 @dataclass(frozen=True)

@@ -1,0 +1,313 @@
+// abi.cu -- host side of the C ABI declared in include/rps.h: argument checks,
+// launch configuration, workspace layout and the device error word.
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include "rps_internal.cuh"
+
+namespace rps {
+namespace {
+
+// Sticky error word of each device (one copy per device context).
+__device__ uint32_t g_device_error;
+
+constexpr int kMaxDevices = 64;
+constexpr size_t kAlign = 256;
+
+struct DeviceInfo {
+    bool ready = false;
+    int sm_count = 0;
+    int blocks[2][2] = {{0, 0}, {0, 0}};  // [dtype][topk]
+    uint32_t *err = nullptr;
+};
+
+std::mutex g_mutex;
+DeviceInfo g_devices[kMaxDevices];
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+rps_status device_info(DeviceInfo *out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RPS_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_mutex);
+    DeviceInfo &d = g_devices[dev];
+    if (!d.ready) {
+        if (cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return RPS_ERR_CUDA;
+        for (int dt = 0; dt < 2; ++dt)
+            for (int tk = 0; tk < 2; ++tk)
+                if (row_stats_occupancy(dt, tk != 0, &d.blocks[dt][tk]) != cudaSuccess || d.blocks[dt][tk] < 1)
+                    return RPS_ERR_CUDA;
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return RPS_ERR_CUDA;
+        d.err = static_cast<uint32_t *>(p);
+        d.ready = true;
+    }
+    *out = d;
+    return RPS_OK;
+}
+
+bool finite(float x) { return std::isfinite(x); }
+
+// Checks the parameters a call uses; `need_search` adds r, tau_pivot, P and K.
+rps_status check_params(const rps_params *p, bool need_search) {
+    if (!p) return RPS_ERR_INVALID_ARG;
+    if (p->k_max < 1) return RPS_ERR_INVALID_ARG;
+    if (p->k_max > RPS_MAX_K) return RPS_ERR_UNSUPPORTED;
+    if (!need_search) return RPS_OK;
+    if (!finite(p->r) || !(p->r > 0.f) || p->r > 1.f) return RPS_ERR_INVALID_ARG;
+    if (!finite(p->tau) || !finite(p->tau_pivot)) return RPS_ERR_INVALID_ARG;
+    if (!finite(p->lambda) || p->lambda < 0.f) return RPS_ERR_INVALID_ARG;
+    if (p->n_pivots < 1 || p->tokens_per_pivot < 1 || p->tokens_per_pivot > p->k_max) return RPS_ERR_INVALID_ARG;
+    if (p->n_pivots > RPS_MAX_PIVOTS) return RPS_ERR_UNSUPPORTED;
+    return RPS_OK;
+}
+
+rps_status check_logits(const rps_logits *l) {
+    if (!l || !l->data) return RPS_ERR_INVALID_ARG;
+    if (l->dtype != RPS_F32 && l->dtype != RPS_BF16) return RPS_ERR_INVALID_ARG;
+    if (l->vocab < 1 || l->vocab > INT32_MAX || l->n_req < 1 || l->n_branch < 1 || l->n_pos < 1)
+        return RPS_ERR_INVALID_ARG;
+    if (l->req_stride < 0 || l->branch_stride < 0 || l->pos_stride < 0) return RPS_ERR_INVALID_ARG;
+    const int64_t esize = l->dtype == RPS_BF16 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(l->data) % 16 != 0) return RPS_ERR_INVALID_ARG;
+    if ((l->req_stride * esize) % 16 || (l->branch_stride * esize) % 16 || (l->pos_stride * esize) % 16)
+        return RPS_ERR_INVALID_ARG;
+    return RPS_OK;
+}
+
+struct WorkspaceLayout {
+    size_t ticket, part, topk, total;
+};
+
+WorkspaceLayout layout(int64_t max_rows, int32_t k) {
+    WorkspaceLayout w;
+    const size_t rows = static_cast<size_t>(max_rows);
+    w.ticket = 0;
+    w.part = align_up(rows * sizeof(uint32_t));
+    w.topk = w.part + align_up(rows * kMaxPartials * sizeof(Partial));
+    w.total = w.topk + (k > 0 ? align_up(rows * kMaxPartials * static_cast<size_t>(k) * sizeof(float2)) : 0);
+    return w;
+}
+
+rps_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RPS_OK : RPS_ERR_CUDA; }
+
+}  // namespace
+}  // namespace rps
+
+using namespace rps;
+
+extern "C" {
+
+size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t k_max) {
+    if (max_rows < 1 || vocab < 1 || k_max < 0 || k_max > RPS_MAX_K) return 0;
+    return layout(max_rows, k_max).total;
+}
+
+rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream) {
+    if (!d_ws || ws_bytes == 0) return RPS_ERR_INVALID_ARG;
+    return from_cuda(cudaMemsetAsync(d_ws, 0, ws_bytes, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                          const rps_row_stats *out, void *d_ws, size_t ws_bytes, rps_stream_t stream) {
+    rps_status st = check_logits(logits);
+    if (st != RPS_OK) return st;
+    if (!rows || (!rows->rows && !rows->mask_pos) || rows->n_seg < 1 || rows->cap < 1) return RPS_ERR_INVALID_ARG;
+    if (rows->n_seg > RPS_MAX_SEGMENTS) return RPS_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(rows->n_seg) * rows->cap > INT32_MAX / 3) return RPS_ERR_INVALID_ARG;
+    if (!out || !out->zmax || !out->lse || !out->H || !out->pmax || !out->argmax) return RPS_ERR_INVALID_ARG;
+    const bool topk = out->topk_idx != nullptr;
+    int32_t k = 0;
+    if (topk) {
+        if ((st = check_params(prm, false)) != RPS_OK) return st;
+        if (!out->topk_logit || !out->mu || !out->htrunc) return RPS_ERR_INVALID_ARG;
+        if (prm->k_max > logits->vocab) return RPS_ERR_INVALID_ARG;
+        k = prm->k_max;
+    }
+    const int64_t max_rows = static_cast<int64_t>(rows->n_seg) * rows->cap;
+    const WorkspaceLayout w = layout(max_rows, k);
+    if (!d_ws || ws_bytes < w.total || reinterpret_cast<uintptr_t>(d_ws) % 16 != 0) return RPS_ERR_INVALID_ARG;
+
+    DeviceInfo dev;
+    if ((st = device_info(&dev)) != RPS_OK) return st;
+    const int esize = logits->dtype == RPS_BF16 ? 2 : 4;
+    const int per_unit = 16 / esize;
+
+    RowStatsArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.data = logits->data;
+    a.vocab = logits->vocab;
+    a.req_stride = logits->req_stride;
+    a.branch_stride = logits->branch_stride;
+    a.pos_stride = logits->pos_stride;
+    a.n_req = logits->n_req;
+    a.n_branch = logits->n_branch;
+    a.n_pos = logits->n_pos;
+    a.rows = rows->rows;
+    a.seg_cnt = rows->seg_cnt;
+    a.n_seg = rows->n_seg;
+    a.cap = rows->cap;
+    a.mask_pos = rows->mask_pos;
+    a.mask_branch = rows->mask_branch;
+    a.k = k;
+    a.zmax = out->zmax;
+    a.lse = out->lse;
+    a.H = out->H;
+    a.pmax = out->pmax;
+    a.argmax = out->argmax;
+    a.mu = out->mu;
+    a.htrunc = out->htrunc;
+    a.topk_idx = out->topk_idx;
+    a.topk_logit = out->topk_logit;
+    char *ws = static_cast<char *>(d_ws);
+    a.ticket = reinterpret_cast<uint32_t *>(ws + w.ticket);
+    a.part = reinterpret_cast<Partial *>(ws + w.part);
+    a.part_topk = k > 0 ? reinterpret_cast<float2 *>(ws + w.topk) : nullptr;
+    a.units_per_row = (logits->vocab + per_unit - 1) / per_unit;
+    const int grid = dev.sm_count * dev.blocks[logits->dtype][topk ? 1 : 0];
+    a.warps = grid * (kRowThreads / 32);
+    a.min_piece = (a.units_per_row + (kMaxPartials - 2) - 1) / (kMaxPartials - 2);
+    a.err = dev.err;
+    return from_cuda(launch_row_stats(a, logits->dtype, grid, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
+                             const int32_t *d_mask_cnt, const rps_params *prm, const rps_pivots *out,
+                             rps_stream_t stream) {
+    rps_status st = check_params(prm, true);
+    if (st != RPS_OK) return st;
+    if (!base || !base->zmax || !base->pmax || !base->argmax || !base->mu || !base->htrunc || !base->topk_idx ||
+        !base->topk_logit)
+        return RPS_ERR_INVALID_ARG;
+    if (n_req < 1 || L < 1 || !d_mask_pos || !d_mask_cnt) return RPS_ERR_INVALID_ARG;
+    if (L > RPS_MAX_POS) return RPS_ERR_UNSUPPORTED;
+    if (!out || !out->n_commit || !out->commit_pos || !out->commit_tok || !out->rem_cnt || !out->rem_k ||
+        !out->rem_pos || !out->state || !out->pivot_k || !out->pivot_pos || !out->n_cand || !out->cand_tok ||
+        !out->branch_valid || !out->branch_off || !out->branch_cnt || !out->n_branch_rows || !out->branch_rows)
+        return RPS_ERR_INVALID_ARG;
+    DeviceInfo dev;
+    if ((st = device_info(&dev)) != RPS_OK) return st;
+    SelectArgs a;
+    a.zmax = base->zmax;
+    a.pmax = base->pmax;
+    a.mu = base->mu;
+    a.htrunc = base->htrunc;
+    a.topk_logit = base->topk_logit;
+    a.argmax = base->argmax;
+    a.topk_idx = base->topk_idx;
+    a.k_max = prm->k_max;
+    a.mask_pos = d_mask_pos;
+    a.mask_cnt = d_mask_cnt;
+    a.n_req = n_req;
+    a.L = L;
+    a.P = prm->n_pivots;
+    a.K = prm->tokens_per_pivot;
+    a.tau = prm->tau;
+    a.tau_pivot = prm->tau_pivot;
+    a.log_r = std::log(static_cast<double>(prm->r));
+    a.out = *out;
+    a.err = dev.err;
+    return from_cuda(launch_select(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_branch,
+                              const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req,
+                              int32_t L, const rps_pivots *piv, const rps_params *prm,
+                              const rps_branch_scores *out, rps_stream_t stream) {
+    rps_status st = check_params(prm, true);
+    if (st != RPS_OK) return st;
+    if ((st = check_logits(anchor_logits)) != RPS_OK) return st;
+    if (anchor_branch < 0 || anchor_branch >= anchor_logits->n_branch) return RPS_ERR_INVALID_ARG;
+    if (n_req < 1 || L < 1 || n_req > anchor_logits->n_req) return RPS_ERR_INVALID_ARG;
+    if (L > RPS_MAX_POS) return RPS_ERR_UNSUPPORTED;
+    if (!anchor || !anchor->zmax || !anchor->lse || !anchor->H || !anchor->pmax) return RPS_ERR_INVALID_ARG;
+    if (!branch || !branch->H || !branch->pmax) return RPS_ERR_INVALID_ARG;
+    if (!piv || !piv->state || !piv->rem_cnt || !piv->rem_k || !piv->pivot_k || !piv->pivot_pos || !piv->n_cand ||
+        !piv->cand_tok || !piv->branch_valid || !piv->branch_off || !piv->branch_cnt)
+        return RPS_ERR_INVALID_ARG;
+    if (!out || !out->mean_H || !out->n_tau || !out->log_a || !out->score) return RPS_ERR_INVALID_ARG;
+    DeviceInfo dev;
+    if ((st = device_info(&dev)) != RPS_OK) return st;
+    ScoreArgs a;
+    a.anchor_data = anchor_logits->data;
+    a.dtype = anchor_logits->dtype;
+    a.vocab = anchor_logits->vocab;
+    a.req_stride = anchor_logits->req_stride;
+    a.pos_stride = anchor_logits->pos_stride;
+    a.branch_offset = static_cast<int64_t>(anchor_branch) * anchor_logits->branch_stride;
+    a.n_pos = anchor_logits->n_pos;
+    a.a_H = anchor->H;
+    a.a_pmax = anchor->pmax;
+    a.a_lse = anchor->lse;
+    a.a_zmax = anchor->zmax;
+    a.b_H = branch->H;
+    a.b_pmax = branch->pmax;
+    a.piv = *piv;
+    a.n_req = n_req;
+    a.L = L;
+    a.P = prm->n_pivots;
+    a.K = prm->tokens_per_pivot;
+    a.lambda = prm->lambda;
+    a.tau = prm->tau;
+    a.out = *out;
+    a.err = dev.err;
+    return from_cuda(launch_score(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
+                      const rps_params *prm, const rps_commit_out *out, rps_stream_t stream) {
+    rps_status st = check_params(prm, true);
+    if (st != RPS_OK) return st;
+    if (!scores || !scores->score || n_req < 1 || L < 1) return RPS_ERR_INVALID_ARG;
+    if (L > RPS_MAX_POS) return RPS_ERR_UNSUPPORTED;
+    if (!piv || !piv->state || !piv->pivot_pos || !piv->n_cand || !piv->cand_tok || !piv->branch_valid ||
+        !piv->rem_cnt || !piv->rem_pos)
+        return RPS_ERR_INVALID_ARG;
+    if (!out || !out->best_slot || !out->gain || !out->winner || !out->commit_pos || !out->commit_tok ||
+        !out->margin || !out->mask_pos || !out->mask_cnt)
+        return RPS_ERR_INVALID_ARG;
+    if (out->mask_pos == piv->rem_pos) return RPS_ERR_INVALID_ARG;
+    DeviceInfo dev;
+    if ((st = device_info(&dev)) != RPS_OK) return st;
+    CommitArgs a;
+    a.score = scores->score;
+    a.piv = *piv;
+    a.n_req = n_req;
+    a.L = L;
+    a.P = prm->n_pivots;
+    a.K = prm->tokens_per_pivot;
+    a.out = *out;
+    return from_cuda(launch_commit(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_poll_device_status(rps_stream_t stream, uint32_t *detail) {
+    if (detail) *detail = 0;
+    if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return RPS_ERR_CUDA;
+    DeviceInfo dev;
+    rps_status st = device_info(&dev);
+    if (st != RPS_OK) return st;
+    uint32_t v = 0;
+    if (cudaMemcpy(&v, dev.err, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return RPS_ERR_CUDA;
+    if (v == 0) return RPS_OK;
+    const uint32_t zero = 0;
+    if (cudaMemcpy(dev.err, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return RPS_ERR_CUDA;
+    if (detail) *detail = v;
+    return RPS_ERR_DEVICE;
+}
+
+const char *rps_status_string(rps_status status) {
+    switch (status) {
+    case RPS_OK: return "RPS_OK";
+    case RPS_ERR_INVALID_ARG: return "RPS_ERR_INVALID_ARG: argument rejected on the host";
+    case RPS_ERR_UNSUPPORTED: return "RPS_ERR_UNSUPPORTED: outside this build's limits";
+    case RPS_ERR_CUDA: return "RPS_ERR_CUDA: a CUDA runtime call failed";
+    case RPS_ERR_DEVICE: return "RPS_ERR_DEVICE: a kernel flagged bad data";
+    case RPS_ERR_TIMEOUT: return "RPS_ERR_TIMEOUT: a bounded device wait gave up";
+    }
+    return "unknown rps_status";
+}
+
+int32_t rps_version(void) { return 100; }
+
+}  // extern "C"

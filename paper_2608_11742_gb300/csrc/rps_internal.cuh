@@ -1,0 +1,124 @@
+// rps_internal.cuh -- declarations shared by the library's translation units.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "rps.h"
+
+namespace rps {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kMaxPartials = 32;   // partial records per row (one merging warp)
+constexpr int kRowThreads = 256;   // threads per block of the row-statistics kernel
+constexpr int kRowMinBlocks = 2;  // resident blocks per SM the register budget must allow
+constexpr int kBatch = 4;          // 16-byte vectors a lane loads per batch
+
+// Partial statistics of one row segment, base-2 online softmax:
+// s = sum 2^u, t = sum u 2^u with u = (z - mref) * log2(e); mx = max z and
+// amax its lowest token index.
+struct __align__(16) Partial {
+    float mref;
+    float s;
+    float t;
+    float mx;
+    int32_t amax;
+    int32_t pad[3];
+};
+
+struct RowStatsArgs {
+    const void *data;
+    int64_t vocab;
+    int64_t req_stride, branch_stride, pos_stride;
+    int32_t n_req, n_branch, n_pos;
+    const int32_t *rows;
+    const int32_t *seg_cnt;
+    int32_t n_seg, cap;
+    const int32_t *mask_pos;  // mask form of the row list when rows == nullptr
+    int32_t mask_branch;
+    int32_t k;  // top-k size, 0 = statistics only
+    // outputs
+    float *zmax, *lse, *H, *pmax, *mu, *htrunc, *topk_logit;
+    int32_t *argmax, *topk_idx;
+    // workspace
+    Partial *part;        // [slots][kMaxPartials]
+    float2 *part_topk;    // [slots][kMaxPartials][k] as (value, index bits)
+    uint32_t *ticket;     // [slots]
+    // decomposition: the rows' 16-byte units are split evenly over `warps` warps
+    int64_t units_per_row;
+    int32_t warps;
+    int64_t min_piece;    // at least ceil(units_per_row / (kMaxPartials - 1))
+    uint32_t *err;
+};
+
+cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, cudaStream_t stream);
+cudaError_t row_stats_occupancy(int dtype, bool topk, int *blocks_per_sm);
+
+struct SelectArgs {
+    // base statistics [q * L + k]
+    const float *zmax, *pmax, *mu, *htrunc, *topk_logit;
+    const int32_t *argmax, *topk_idx;
+    int32_t k_max;
+    const int32_t *mask_pos, *mask_cnt;
+    int32_t n_req, L, P, K;
+    float tau, tau_pivot;
+    double log_r;
+    rps_pivots out;
+    uint32_t *err;
+};
+
+struct ScoreArgs {
+    const void *anchor_data;
+    int32_t dtype;
+    int64_t vocab, req_stride, pos_stride, branch_offset;
+    int32_t n_pos;
+    const float *a_H, *a_pmax, *a_lse, *a_zmax;  // anchor statistics [q * L + k]
+    const float *b_H, *b_pmax;                   // branch statistics, compact [q * NB * L + i]
+    rps_pivots piv;
+    int32_t n_req, L, P, K;
+    float lambda, tau;
+    rps_branch_scores out;
+    uint32_t *err;
+};
+
+struct CommitArgs {
+    const float *score;
+    rps_pivots piv;
+    int32_t n_req, L, P, K;
+    rps_commit_out out;
+};
+
+cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream);
+cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream);
+cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream);
+
+// ---------------------------------------------------------------- device
+__device__ __forceinline__ void flag_error(uint32_t *err, uint32_t bits) {
+    if (err) atomicOr(err, bits);
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFull, v, o));
+    return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+__device__ __forceinline__ int warp_sum_int(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+__device__ __forceinline__ int warp_min_int(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(kFull, v, o));
+    return v;
+}
+
+}  // namespace rps

@@ -1,0 +1,342 @@
+"""ctypes binding of ``librps.so`` (declared in ``include/rps.h``).
+
+Argument marshalling only: each function takes torch CUDA tensors, passes their
+device pointers and the current stream to the C ABI function of the same name,
+and raises ``RPSError`` on a non-OK status. Every step of the scoring path runs
+in the library's CUDA kernels; there is no fallback. Importing this module
+raises ImportError when the library has not been built.
+
+Buffers (``RowStatsBuf``, ``PivotsBuf``, ``ScoresBuf``, ``CommitBuf``) are
+allocated once by the caller and reused; ``Step`` strings the five calls of
+one decoding step together on preallocated buffers.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from dataclasses import dataclass, fields
+from pathlib import Path
+from typing import Optional
+
+import torch
+
+LIB_PATH = Path(__file__).resolve().parent / "librps.so"
+if not LIB_PATH.exists():
+    raise ImportError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+_lib = C.CDLL(str(LIB_PATH))
+
+RPS_OK, RPS_ERR_INVALID_ARG, RPS_ERR_UNSUPPORTED, RPS_ERR_CUDA, RPS_ERR_DEVICE, RPS_ERR_TIMEOUT = range(6)
+RPS_F32, RPS_BF16 = 0, 1
+STATE_SEARCH, STATE_DONE, STATE_NO_FEASIBLE, STATE_NO_CANDIDATES = 0, 1, 2, 3
+WIN_ANCHOR, WIN_SKIP, WIN_DONE = -1, -2, -3
+DEVERR_ROW_INDEX, DEVERR_NONFINITE, DEVERR_MASK, DEVERR_TOKEN = 0x1, 0x2, 0x4, 0x8
+
+_p = C.c_void_p
+
+
+class RpsParams(C.Structure):
+    _fields_ = [("k_max", C.c_int32), ("r", C.c_float), ("tau_pivot", C.c_float), ("tau", C.c_float),
+                ("lambda_", C.c_float), ("n_pivots", C.c_int32), ("tokens_per_pivot", C.c_int32)]
+
+
+class RpsLogits(C.Structure):
+    _fields_ = [("data", _p), ("dtype", C.c_int32), ("n_req", C.c_int32), ("n_branch", C.c_int32),
+                ("n_pos", C.c_int32), ("vocab", C.c_int64), ("req_stride", C.c_int64),
+                ("branch_stride", C.c_int64), ("pos_stride", C.c_int64)]
+
+
+class RpsRowList(C.Structure):
+    _fields_ = [("rows", _p), ("seg_cnt", _p), ("n_seg", C.c_int32), ("cap", C.c_int32),
+                ("mask_pos", _p), ("mask_branch", C.c_int32)]
+
+
+class RpsRowStats(C.Structure):
+    _fields_ = [(n, _p) for n in ("zmax", "lse", "H", "pmax", "argmax", "mu", "htrunc", "topk_idx", "topk_logit")]
+
+
+_PIVOT_FIELDS = ("n_commit", "commit_pos", "commit_tok", "rem_cnt", "rem_k", "rem_pos", "state", "pivot_k",
+                 "pivot_pos", "n_cand", "cand_tok", "branch_valid", "branch_off", "branch_cnt", "n_branch_rows",
+                 "branch_rows")
+
+
+class RpsPivots(C.Structure):
+    _fields_ = [(n, _p) for n in _PIVOT_FIELDS]
+
+
+class RpsBranchScores(C.Structure):
+    _fields_ = [(n, _p) for n in ("mean_H", "n_tau", "log_a", "score")]
+
+
+class RpsCommitOut(C.Structure):
+    _fields_ = [(n, _p) for n in ("best_slot", "gain", "winner", "commit_pos", "commit_tok", "margin", "mask_pos",
+                                  "mask_cnt")]
+
+
+_lib.rps_workspace_bytes.restype = C.c_size_t
+_lib.rps_workspace_bytes.argtypes = [C.c_int64, C.c_int64, C.c_int32]
+_lib.rps_workspace_init.restype = C.c_int
+_lib.rps_workspace_init.argtypes = [_p, C.c_size_t, _p]
+_lib.rps_score_step.restype = C.c_int
+_lib.rps_score_step.argtypes = [C.POINTER(RpsLogits), C.POINTER(RpsRowList), C.POINTER(RpsParams),
+                                C.POINTER(RpsRowStats), _p, C.c_size_t, _p]
+_lib.rps_select_pivots.restype = C.c_int
+_lib.rps_select_pivots.argtypes = [C.POINTER(RpsRowStats), C.c_int32, C.c_int32, _p, _p, C.POINTER(RpsParams),
+                                   C.POINTER(RpsPivots), _p]
+_lib.rps_score_branches.restype = C.c_int
+_lib.rps_score_branches.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.POINTER(RpsRowStats),
+                                    C.POINTER(RpsRowStats), C.c_int32, C.c_int32, C.POINTER(RpsPivots),
+                                    C.POINTER(RpsParams), C.POINTER(RpsBranchScores), _p]
+_lib.rps_commit.restype = C.c_int
+_lib.rps_commit.argtypes = [C.POINTER(RpsBranchScores), C.c_int32, C.c_int32, C.POINTER(RpsPivots),
+                            C.POINTER(RpsParams), C.POINTER(RpsCommitOut), _p]
+_lib.rps_poll_device_status.restype = C.c_int
+_lib.rps_poll_device_status.argtypes = [_p, C.POINTER(C.c_uint32)]
+_lib.rps_status_string.restype = C.c_char_p
+_lib.rps_status_string.argtypes = [C.c_int]
+_lib.rps_version.restype = C.c_int32
+_lib.rps_version.argtypes = []
+
+
+class RPSError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {_lib.rps_status_string(status).decode()}")
+
+
+def _check(status: int, where: str) -> None:
+    if status != RPS_OK:
+        raise RPSError(status, where)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def params(p) -> RpsParams:
+    """C struct from any object with the ``configs.Params`` fields."""
+    return RpsParams(p.k_max, p.r, p.tau_pivot, p.tau, p.lam, p.n_pivots, p.tokens_per_pivot)
+
+
+def logits_desc(t: torch.Tensor) -> RpsLogits:
+    """Descriptor of a ``[n_req][n_branch][n_pos][vocab]`` bf16 / fp32 CUDA tensor."""
+    if t.dim() != 4 or t.stride(3) != 1:
+        raise ValueError("logits must be 4-D with a contiguous vocab dimension")
+    if t.dtype == torch.bfloat16:
+        dt = RPS_BF16
+    elif t.dtype == torch.float32:
+        dt = RPS_F32
+    else:
+        raise TypeError(f"logits must be bf16 or fp32, got {t.dtype}")
+    n_req, nb, L, V = t.shape
+    return RpsLogits(t.data_ptr(), dt, n_req, nb, L, V, t.stride(0), t.stride(1), t.stride(2))
+
+
+# --------------------------------------------------------------------------- buffers
+@dataclass
+class RowStatsBuf:
+    zmax: torch.Tensor
+    lse: torch.Tensor
+    H: torch.Tensor
+    pmax: torch.Tensor
+    argmax: torch.Tensor
+    mu: Optional[torch.Tensor] = None
+    htrunc: Optional[torch.Tensor] = None
+    topk_idx: Optional[torch.Tensor] = None
+    topk_logit: Optional[torch.Tensor] = None
+
+    @staticmethod
+    def alloc(n: int, k: int, device) -> "RowStatsBuf":
+        f = lambda *s: torch.full(s, float("nan"), dtype=torch.float32, device=device)
+        i = lambda *s: torch.full(s, -1, dtype=torch.int32, device=device)
+        if k > 0:
+            return RowStatsBuf(f(n), f(n), f(n), f(n), i(n), f(n), f(n), i(n, k), f(n, k))
+        return RowStatsBuf(f(n), f(n), f(n), f(n), i(n))
+
+    def c(self) -> RpsRowStats:
+        return RpsRowStats(*(_ptr(getattr(self, f.name)) for f in fields(self)))
+
+
+@dataclass
+class PivotsBuf:
+    n_commit: torch.Tensor
+    commit_pos: torch.Tensor
+    commit_tok: torch.Tensor
+    rem_cnt: torch.Tensor
+    rem_k: torch.Tensor
+    rem_pos: torch.Tensor
+    state: torch.Tensor
+    pivot_k: torch.Tensor
+    pivot_pos: torch.Tensor
+    n_cand: torch.Tensor
+    cand_tok: torch.Tensor
+    branch_valid: torch.Tensor
+    branch_off: torch.Tensor
+    branch_cnt: torch.Tensor
+    n_branch_rows: torch.Tensor
+    branch_rows: torch.Tensor
+
+    @staticmethod
+    def alloc(n_req: int, L: int, P: int, K: int, device) -> "PivotsBuf":
+        i = lambda *s: torch.full(s, -1, dtype=torch.int32, device=device)
+        NB = P * K
+        return PivotsBuf(i(n_req), i(n_req, L), i(n_req, L), i(n_req), i(n_req, L), i(n_req, L), i(n_req),
+                         i(n_req, P), i(n_req, P), i(n_req, P), i(n_req, P, K),
+                         torch.zeros(n_req, NB, dtype=torch.uint8, device=device), i(n_req, NB), i(n_req, NB),
+                         i(n_req), i(n_req, NB * L, 3))
+
+    def c(self) -> RpsPivots:
+        return RpsPivots(*(_ptr(getattr(self, n)) for n in _PIVOT_FIELDS))
+
+
+@dataclass
+class ScoresBuf:
+    mean_H: torch.Tensor
+    n_tau: torch.Tensor
+    log_a: torch.Tensor
+    score: torch.Tensor
+
+    @staticmethod
+    def alloc(n_req: int, P: int, K: int, device) -> "ScoresBuf":
+        f = lambda: torch.full((n_req, P, K + 1), float("nan"), dtype=torch.float32, device=device)
+        return ScoresBuf(f(), torch.full((n_req, P, K + 1), -1, dtype=torch.int32, device=device), f(), f())
+
+    def c(self) -> RpsBranchScores:
+        return RpsBranchScores(*(_ptr(getattr(self, f.name)) for f in fields(self)))
+
+
+@dataclass
+class CommitBuf:
+    best_slot: torch.Tensor
+    gain: torch.Tensor
+    winner: torch.Tensor
+    commit_pos: torch.Tensor
+    commit_tok: torch.Tensor
+    margin: torch.Tensor
+    mask_pos: torch.Tensor
+    mask_cnt: torch.Tensor
+
+    @staticmethod
+    def alloc(n_req: int, L: int, P: int, device) -> "CommitBuf":
+        i = lambda *s: torch.full(s, -1, dtype=torch.int32, device=device)
+        f = lambda *s: torch.full(s, float("nan"), dtype=torch.float32, device=device)
+        return CommitBuf(i(n_req, P), f(n_req, P), i(n_req), i(n_req), i(n_req), f(n_req), i(n_req, L), i(n_req))
+
+    def c(self) -> RpsCommitOut:
+        return RpsCommitOut(*(_ptr(getattr(self, f.name)) for f in fields(self)))
+
+
+# --------------------------------------------------------------------------- ABI calls
+def rps_version() -> int:
+    return _lib.rps_version()
+
+
+def rps_status_string(status: int) -> str:
+    return _lib.rps_status_string(status).decode()
+
+
+def rps_workspace_bytes(max_rows: int, vocab: int, k_max: int) -> int:
+    n = _lib.rps_workspace_bytes(max_rows, vocab, k_max)
+    if n == 0:
+        raise RPSError(RPS_ERR_INVALID_ARG, "rps_workspace_bytes")
+    return n
+
+
+def rps_workspace_init(ws: torch.Tensor, stream=None) -> None:
+    _check(_lib.rps_workspace_init(ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)),
+           "rps_workspace_init")
+
+
+def rps_score_step(logits: torch.Tensor, rows: Optional[torch.Tensor], seg_cnt: Optional[torch.Tensor], n_seg: int,
+                   cap: int, prm, out: RowStatsBuf, ws: torch.Tensor, stream=None,
+                   mask_pos: Optional[torch.Tensor] = None, mask_branch: int = 0) -> None:
+    desc = logits_desc(logits)
+    rl = RpsRowList(_ptr(rows), _ptr(seg_cnt), n_seg, cap, _ptr(mask_pos), mask_branch)
+    p = params(prm)
+    st = out.c()
+    _check(_lib.rps_score_step(C.byref(desc), C.byref(rl), C.byref(p), C.byref(st), ws.data_ptr(),
+                               ws.numel() * ws.element_size(), _stream(stream)), "rps_score_step")
+
+
+def rps_select_pivots(base: RowStatsBuf, n_req: int, L: int, mask_pos: torch.Tensor, mask_cnt: torch.Tensor, prm,
+                      out: PivotsBuf, stream=None) -> None:
+    b, p, o = base.c(), params(prm), out.c()
+    _check(_lib.rps_select_pivots(C.byref(b), n_req, L, mask_pos.data_ptr(), mask_cnt.data_ptr(), C.byref(p),
+                                  C.byref(o), _stream(stream)), "rps_select_pivots")
+
+
+def rps_score_branches(anchor_logits: torch.Tensor, anchor_branch: int, anchor: RowStatsBuf, branch: RowStatsBuf,
+                       n_req: int, L: int, piv: PivotsBuf, prm, out: ScoresBuf, stream=None) -> None:
+    d, a, b, pv, p, o = logits_desc(anchor_logits), anchor.c(), branch.c(), piv.c(), params(prm), out.c()
+    _check(_lib.rps_score_branches(C.byref(d), anchor_branch, C.byref(a), C.byref(b), n_req, L, C.byref(pv),
+                                   C.byref(p), C.byref(o), _stream(stream)), "rps_score_branches")
+
+
+def rps_commit(scores: ScoresBuf, n_req: int, L: int, piv: PivotsBuf, prm, out: CommitBuf, stream=None) -> None:
+    s, pv, p, o = scores.c(), piv.c(), params(prm), out.c()
+    _check(_lib.rps_commit(C.byref(s), n_req, L, C.byref(pv), C.byref(p), C.byref(o), _stream(stream)),
+           "rps_commit")
+
+
+def rps_poll_device_status(stream=None):
+    """Synchronise and return (status, detail bits); clears the device error word."""
+    detail = C.c_uint32(0)
+    st = _lib.rps_poll_device_status(_stream(stream), C.byref(detail))
+    return st, detail.value
+
+
+# --------------------------------------------------------------------------- one step
+class Step:
+    """Preallocated buffers and the five ABI calls of one RPS decoding step.
+
+    The base branch (0) of ``logits`` is the anchor, as in the workloads here.
+    Kernels launched per ``run``: row statistics of the masked base rows (top-k
+    mode), pivot selection, row statistics of the lookahead rows, branch
+    scores, commit.
+    """
+    LAUNCHES = 5
+
+    def __init__(self, n_req: int, L: int, V: int, prm, device):
+        self.n_req, self.L, self.V, self.prm = n_req, L, V, prm
+        P, K, k = prm.n_pivots, prm.tokens_per_pivot, prm.k_max
+        self.NB = P * K
+        self.base = RowStatsBuf.alloc(n_req * L, k, device)
+        self.branch = RowStatsBuf.alloc(n_req * self.NB * L, 0, device)
+        self.piv = PivotsBuf.alloc(n_req, L, P, K, device)
+        self.scores = ScoresBuf.alloc(n_req, P, K, device)
+        self.commit = CommitBuf.alloc(n_req, L, P, device)
+        base_ws = rps_workspace_bytes(n_req * L, V, k)
+        br_ws = rps_workspace_bytes(n_req * self.NB * L, V, 0)
+        self.ws_base = torch.empty(base_ws, dtype=torch.uint8, device=device)
+        self.ws_branch = torch.empty(br_ws, dtype=torch.uint8, device=device)
+        rps_workspace_init(self.ws_base)
+        rps_workspace_init(self.ws_branch)
+
+    def score_base(self, logits, mask_pos, mask_cnt, stream=None):
+        rps_score_step(logits, None, mask_cnt, self.n_req, self.L, self.prm, self.base, self.ws_base, stream,
+                       mask_pos=mask_pos, mask_branch=0)
+
+    def select(self, mask_pos, mask_cnt, stream=None):
+        rps_select_pivots(self.base, self.n_req, self.L, mask_pos, mask_cnt, self.prm, self.piv, stream)
+
+    def score_branch_rows(self, logits, stream=None):
+        rps_score_step(logits, self.piv.branch_rows, self.piv.n_branch_rows, self.n_req, self.NB * self.L, self.prm,
+                       self.branch, self.ws_branch, stream)
+
+    def score(self, logits, stream=None):
+        rps_score_branches(logits, 0, self.base, self.branch, self.n_req, self.L, self.piv, self.prm, self.scores,
+                           stream)
+
+    def decide(self, stream=None):
+        rps_commit(self.scores, self.n_req, self.L, self.piv, self.prm, self.commit, stream)
+
+    def run(self, logits, mask_pos, mask_cnt, stream=None):
+        self.score_base(logits, mask_pos, mask_cnt, stream)
+        self.select(mask_pos, mask_cnt, stream)
+        self.score_branch_rows(logits, stream)
+        self.score(logits, stream)
+        self.decide(stream)

@@ -233,3 +233,48 @@ def ragged_count(seed: int, req: int, lo: int, hi: int) -> int:
     """Masked count of request ``req`` drawn uniformly from [lo, hi]."""
     x0 = int(philox4x32_10(req, 0, 0, _tag(TAG_COUNT), seed, KEY1)[0])
     return lo + x0 % (hi - lo + 1)
+
+
+# ---------------------------------------------------------------------------
+# Device twin (librps_synth.so): the same bits, written straight into HBM.
+# ---------------------------------------------------------------------------
+_SYNTH_LIB = None
+
+
+def _synth_lib():
+    global _SYNTH_LIB
+    if _SYNTH_LIB is None:
+        import ctypes as C
+        from pathlib import Path
+        path = Path(__file__).resolve().parent / "librps_synth.so"
+        if not path.exists():
+            raise ImportError(f"{path} is missing: build the CUDA libraries first")
+        lib = C.CDLL(str(path))
+        lib.rps_synth_fill.restype = C.c_int32
+        lib.rps_synth_fill.argtypes = [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int64,
+                                       C.c_int64, C.c_int64, C.c_int64, C.c_uint32, C.c_uint64, C.c_uint64,
+                                       C.c_uint32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
+        _SYNTH_LIB = lib
+    return _SYNTH_LIB
+
+
+def device_fill(out, seed: int, mixture, step: int = 0, scale=None, epoch=None, valid=None, stream=None) -> None:
+    """Fill a CUDA tensor ``[n_req][1 + n_branch][L][V]`` (bf16 or fp32) on the device.
+
+    ``scale`` (float32), ``epoch`` (int32) and ``valid`` (uint8) are optional
+    ``[n_req][L]`` CUDA tensors with the meaning of ``make_logits``.
+    """
+    import torch
+    if out.dim() != 4 or out.stride(3) != 1:
+        raise ValueError("out must be 4-D with a contiguous last dimension")
+    dtype = {torch.bfloat16: 1, torch.float32: 0}[out.dtype]
+    n_req, nb1, L, V = out.shape
+    t_low, t_mid = regime_thresholds(mixture)
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    ptr = lambda t: None if t is None else t.data_ptr()
+    rc = _synth_lib().rps_synth_fill(out.data_ptr(), dtype, n_req, nb1 - 1, L, V, out.stride(0), out.stride(1),
+                                     out.stride(2), seed, t_low, t_mid, step, ptr(scale), ptr(epoch), ptr(valid),
+                                     stream.cuda_stream)
+    if rc != 0:
+        raise RuntimeError(f"rps_synth_fill failed with code {rc}")
