@@ -255,6 +255,31 @@ rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_br
 rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
                       const rps_params *prm, const rps_commit_out *out, rps_stream_t stream);
 
+/* Bytes of scratch the library holds on each device for rps_score_step_noalloc. */
+#define RPS_STATIC_SCRATCH_BYTES (8u << 20)
+
+/*
+ * rps_score_step without a caller workspace. The paper has no counterpart: this
+ * is a deployment variant for callers that cannot allocate device memory, such
+ * as plugins of a host runtime that owns every device allocation and forbids
+ * others, or bindings from languages with no CUDA allocator. Inputs and outputs
+ * are as for rps_score_step; the scratch is a fixed RPS_STATIC_SCRATCH_BYTES
+ * array inside the library, which every GPU that loads the library keeps until
+ * the process exits.
+ *   - Requests whose rps_workspace_bytes(n_seg * cap, vocab, k) exceeds
+ *     RPS_STATIC_SCRATCH_BYTES return RPS_ERR_UNSUPPORTED before anything is
+ *     enqueued; argument errors return RPS_ERR_INVALID_ARG likewise.
+ *   - No cudaMalloc, cudaFree or other allocating call is made. Each call clears
+ *     the part of the array it uses with cudaMemsetAsync on `stream`.
+ *   - The first call on each device looks up the array's device address while
+ *     that device is current; make that first call before any stream capture.
+ *   - All calls on a device share the one array: calls that can overlap on the
+ *     GPU (different streams without ordering between them) race and corrupt each
+ *     other's results. Order them on one stream or serialise them.
+ */
+rps_status rps_score_step_noalloc(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                                  const rps_row_stats *out, rps_stream_t stream);
+
 /* Synchronise `stream`, then read and clear the calling device's error word.
  * Returns RPS_OK or RPS_ERR_DEVICE (with the RPS_DEVERR_* bits in *detail when
  * detail != NULL), or RPS_ERR_CUDA if the synchronisation itself failed. */

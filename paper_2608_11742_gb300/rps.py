@@ -78,6 +78,9 @@ _lib.rps_workspace_init.argtypes = [_p, C.c_size_t, _p]
 _lib.rps_score_step.restype = C.c_int
 _lib.rps_score_step.argtypes = [C.POINTER(RpsLogits), C.POINTER(RpsRowList), C.POINTER(RpsParams),
                                 C.POINTER(RpsRowStats), _p, C.c_size_t, _p]
+_lib.rps_score_step_noalloc.restype = C.c_int
+_lib.rps_score_step_noalloc.argtypes = [C.POINTER(RpsLogits), C.POINTER(RpsRowList), C.POINTER(RpsParams),
+                                        C.POINTER(RpsRowStats), _p]
 _lib.rps_select_pivots.restype = C.c_int
 _lib.rps_select_pivots.argtypes = [C.POINTER(RpsRowStats), C.c_int32, C.c_int32, _p, _p, C.POINTER(RpsParams),
                                    C.POINTER(RpsPivots), _p]
@@ -260,6 +263,19 @@ def rps_score_step(logits: torch.Tensor, rows: Optional[torch.Tensor], seg_cnt: 
     st = out.c()
     _check(_lib.rps_score_step(C.byref(desc), C.byref(rl), C.byref(p), C.byref(st), ws.data_ptr(),
                                ws.numel() * ws.element_size(), _stream(stream)), "rps_score_step")
+
+
+def rps_score_step_noalloc(logits: torch.Tensor, rows: Optional[torch.Tensor], seg_cnt: Optional[torch.Tensor],
+                           n_seg: int, cap: int, prm, out: RowStatsBuf, stream=None,
+                           mask_pos: Optional[torch.Tensor] = None, mask_branch: int = 0) -> None:
+    """rps_score_step with the library's fixed scratch instead of a caller workspace,
+    for callers that cannot allocate device memory (see include/rps.h)."""
+    desc = logits_desc(logits)
+    rl = RpsRowList(_ptr(rows), _ptr(seg_cnt), n_seg, cap, _ptr(mask_pos), mask_branch)
+    p = params(prm)
+    st = out.c()
+    _check(_lib.rps_score_step_noalloc(C.byref(desc), C.byref(rl), C.byref(p), C.byref(st), _stream(stream)),
+           "rps_score_step_noalloc")
 
 
 def rps_select_pivots(base: RowStatsBuf, n_req: int, L: int, mask_pos: torch.Tensor, mask_cnt: torch.Tensor, prm,
