@@ -128,7 +128,7 @@ class Workload:
         mpos, mcnt = w.mask()
         self.mpos = torch.from_numpy(mpos).to(device)
         self.mcnt = torch.from_numpy(mcnt).to(device)
-        self.step = rps.Step(w.n_req, w.L, w.V, prm, device)
+        self.step = rps.Step(w.n_req, w.L, w.V, prm, device, dt)
         self.stream = torch.cuda.Stream(device)
         self.ev = None
         with torch.cuda.stream(self.stream):
@@ -156,8 +156,7 @@ class Workload:
             self.step.score_branch_rows(self.logits)
             if ev:
                 ev[1].record()
-            self.step.score(self.logits)
-            self.step.decide()
+            self.step.score_and_decide(self.logits)
         self.ev = ev
         if ev is None:
             self.k1_graph = torch.cuda.CUDAGraph()

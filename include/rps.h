@@ -59,7 +59,7 @@ typedef enum {
     RPS_ERR_UNSUPPORTED = 2, /* well-formed request outside this build's limits */
     RPS_ERR_CUDA = 3,        /* a CUDA runtime call (launch, attribute query) failed */
     RPS_ERR_DEVICE = 4,      /* a kernel flagged bad data; see rps_poll_device_status */
-    RPS_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up (no kernel here waits) */
+    RPS_ERR_TIMEOUT = 5      /* reserved; a kernel wait that gives up is reported as RPS_DEVERR_TIMEOUT */
 } rps_status;
 
 /* Bits of the device error word. */
@@ -67,6 +67,8 @@ typedef enum {
 #define RPS_DEVERR_NONFINITE 0x2u  /* a scored row holds NaN or no finite logit */
 #define RPS_DEVERR_MASK 0x4u       /* mask count above capacity or position out of range */
 #define RPS_DEVERR_TOKEN 0x8u      /* candidate token outside the vocabulary */
+#define RPS_DEVERR_TIMEOUT 0x10u   /* a bounded wait for an asynchronous copy gave up; the call's
+                                      outputs are incomplete and its workspace must be re-zeroed */
 
 typedef enum { RPS_F32 = 0, RPS_BF16 = 1 } rps_dtype;
 
@@ -185,9 +187,9 @@ typedef struct {
 } rps_commit_out;
 
 /* Bytes of workspace rps_score_step needs for up to max_rows row slots
- * (n_seg * cap) of `vocab` logits with top-k size k_max (0 for statistics
- * only). Returns 0 for invalid arguments. */
-size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t k_max);
+ * (n_seg * cap) of `vocab` logits of the given rps_dtype with top-k size k_max
+ * (0 for statistics only). Returns 0 for invalid arguments. */
+size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k_max);
 
 /* Zero a workspace (asynchronously on `stream`). A workspace must be zeroed
  * once before its first use; every completed rps_score_step leaves it ready
@@ -202,7 +204,7 @@ rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream);
  * fp32 arithmetic; argmax and T_i are exact (taken on the input values).
  * Errors: RPS_ERR_INVALID_ARG for NULL pointers, a misaligned tensor, sizes out
  * of range or a workspace smaller than rps_workspace_bytes(n_seg * cap, vocab,
- * k); RPS_ERR_UNSUPPORTED above RPS_MAX_K / RPS_MAX_SEGMENTS.
+ * dtype, k); RPS_ERR_UNSUPPORTED above RPS_MAX_K / RPS_MAX_SEGMENTS.
  */
 rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
                           const rps_row_stats *out, void *d_ws, size_t ws_bytes, rps_stream_t stream);
@@ -255,6 +257,13 @@ rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_br
 rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
                       const rps_params *prm, const rps_commit_out *out, rps_stream_t stream);
 
+/* rps_score_branches followed by rps_commit in one launch (same arguments and
+ * results as the two calls in sequence). */
+rps_status rps_score_and_commit(const rps_logits *anchor_logits, int32_t anchor_branch,
+                                const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req, int32_t L,
+                                const rps_pivots *piv, const rps_params *prm, const rps_branch_scores *scores,
+                                const rps_commit_out *out, rps_stream_t stream);
+
 /* Bytes of scratch the library holds on each device for rps_score_step_noalloc. */
 #define RPS_STATIC_SCRATCH_BYTES (8u << 20)
 
@@ -266,7 +275,7 @@ rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L,
  * are as for rps_score_step; the scratch is a fixed RPS_STATIC_SCRATCH_BYTES
  * array inside the library, which every GPU that loads the library keeps until
  * the process exits.
- *   - Requests whose rps_workspace_bytes(n_seg * cap, vocab, k) exceeds
+ *   - Requests whose rps_workspace_bytes(n_seg * cap, vocab, dtype, k) exceeds
  *     RPS_STATIC_SCRATCH_BYTES return RPS_ERR_UNSUPPORTED before anything is
  *     enqueued; argument errors return RPS_ERR_INVALID_ARG likewise.
  *   - No cudaMalloc, cudaFree or other allocating call is made. Each call clears

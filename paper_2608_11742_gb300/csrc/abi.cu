@@ -77,16 +77,21 @@ rps_status check_logits(const rps_logits *l) {
 }
 
 struct WorkspaceLayout {
-    size_t ticket, part, topk, total;
+    size_t ticket, part, topk, sketch, total;
 };
 
-WorkspaceLayout layout(int64_t max_rows, int32_t k) {
+// Tickets, partial records, per-piece top-k lists and the top-k sketch (one
+// element-sized entry per 16-byte unit of each row, of which a quarter is used).
+WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k) {
     WorkspaceLayout w;
     const size_t rows = static_cast<size_t>(max_rows);
+    const size_t esize = dtype == RPS_BF16 ? 2 : 4;
+    const size_t units = (static_cast<size_t>(vocab) * esize + 15) / 16;
     w.ticket = 0;
     w.part = align_up(rows * sizeof(uint32_t));
     w.topk = w.part + align_up(rows * kMaxPartials * sizeof(Partial));
-    w.total = w.topk + (k > 0 ? align_up(rows * kMaxPartials * static_cast<size_t>(k) * sizeof(float2)) : 0);
+    w.sketch = w.topk + (k > 0 ? align_up(rows * kMaxPartials * static_cast<size_t>(k) * sizeof(float2)) : 0);
+    w.total = w.sketch + (k > 0 ? align_up(rows * units * esize) : 0);
     return w;
 }
 
@@ -99,9 +104,10 @@ using namespace rps;
 
 extern "C" {
 
-size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t k_max) {
+size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k_max) {
     if (max_rows < 1 || vocab < 1 || k_max < 0 || k_max > RPS_MAX_K) return 0;
-    return layout(max_rows, k_max).total;
+    if (dtype != RPS_F32 && dtype != RPS_BF16) return 0;
+    return layout(max_rows, vocab, dtype, k_max).total;
 }
 
 rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream) {
@@ -126,7 +132,7 @@ rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, co
         k = prm->k_max;
     }
     const int64_t max_rows = static_cast<int64_t>(rows->n_seg) * rows->cap;
-    const WorkspaceLayout w = layout(max_rows, k);
+    const WorkspaceLayout w = layout(max_rows, logits->vocab, logits->dtype, k);
     if (!d_ws || ws_bytes < w.total || reinterpret_cast<uintptr_t>(d_ws) % 16 != 0) return RPS_ERR_INVALID_ARG;
 
     DeviceInfo dev;
@@ -164,6 +170,7 @@ rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, co
     a.ticket = reinterpret_cast<uint32_t *>(ws + w.ticket);
     a.part = reinterpret_cast<Partial *>(ws + w.part);
     a.part_topk = k > 0 ? reinterpret_cast<float2 *>(ws + w.topk) : nullptr;
+    a.sketch = k > 0 ? static_cast<void *>(ws + w.sketch) : nullptr;
     a.units_per_row = (logits->vocab + per_unit - 1) / per_unit;
     const int grid = dev.sm_count * dev.blocks[logits->dtype][topk ? 1 : 0];
     a.warps = grid * (kRowThreads / 32);
@@ -211,10 +218,14 @@ rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L
     return from_cuda(launch_select(a, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_branch,
-                              const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req,
-                              int32_t L, const rps_pivots *piv, const rps_params *prm,
-                              const rps_branch_scores *out, rps_stream_t stream) {
+}  // extern "C"
+
+namespace rps {
+namespace {
+
+rps_status make_score_args(const rps_logits *anchor_logits, int32_t anchor_branch, const rps_row_stats *anchor,
+                           const rps_row_stats *branch, int32_t n_req, int32_t L, const rps_pivots *piv,
+                           const rps_params *prm, const rps_branch_scores *out, ScoreArgs *a) {
     rps_status st = check_params(prm, true);
     if (st != RPS_OK) return st;
     if ((st = check_logits(anchor_logits)) != RPS_OK) return st;
@@ -227,36 +238,33 @@ rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_br
         !piv->cand_tok || !piv->branch_valid || !piv->branch_off || !piv->branch_cnt)
         return RPS_ERR_INVALID_ARG;
     if (!out || !out->mean_H || !out->n_tau || !out->log_a || !out->score) return RPS_ERR_INVALID_ARG;
-    DeviceInfo dev;
-    if ((st = device_info(&dev)) != RPS_OK) return st;
-    ScoreArgs a;
-    a.anchor_data = anchor_logits->data;
-    a.dtype = anchor_logits->dtype;
-    a.vocab = anchor_logits->vocab;
-    a.req_stride = anchor_logits->req_stride;
-    a.pos_stride = anchor_logits->pos_stride;
-    a.branch_offset = static_cast<int64_t>(anchor_branch) * anchor_logits->branch_stride;
-    a.n_pos = anchor_logits->n_pos;
-    a.a_H = anchor->H;
-    a.a_pmax = anchor->pmax;
-    a.a_lse = anchor->lse;
-    a.a_zmax = anchor->zmax;
-    a.b_H = branch->H;
-    a.b_pmax = branch->pmax;
-    a.piv = *piv;
-    a.n_req = n_req;
-    a.L = L;
-    a.P = prm->n_pivots;
-    a.K = prm->tokens_per_pivot;
-    a.lambda = prm->lambda;
-    a.tau = prm->tau;
-    a.out = *out;
-    a.err = dev.err;
-    return from_cuda(launch_score(a, reinterpret_cast<cudaStream_t>(stream)));
+    a->anchor_data = anchor_logits->data;
+    a->dtype = anchor_logits->dtype;
+    a->vocab = anchor_logits->vocab;
+    a->req_stride = anchor_logits->req_stride;
+    a->pos_stride = anchor_logits->pos_stride;
+    a->branch_offset = static_cast<int64_t>(anchor_branch) * anchor_logits->branch_stride;
+    a->n_pos = anchor_logits->n_pos;
+    a->a_H = anchor->H;
+    a->a_pmax = anchor->pmax;
+    a->a_lse = anchor->lse;
+    a->a_zmax = anchor->zmax;
+    a->b_H = branch->H;
+    a->b_pmax = branch->pmax;
+    a->piv = *piv;
+    a->n_req = n_req;
+    a->L = L;
+    a->P = prm->n_pivots;
+    a->K = prm->tokens_per_pivot;
+    a->lambda = prm->lambda;
+    a->tau = prm->tau;
+    a->out = *out;
+    a->err = nullptr;
+    return RPS_OK;
 }
 
-rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
-                      const rps_params *prm, const rps_commit_out *out, rps_stream_t stream) {
+rps_status make_commit_args(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
+                            const rps_params *prm, const rps_commit_out *out, CommitArgs *a) {
     rps_status st = check_params(prm, true);
     if (st != RPS_OK) return st;
     if (!scores || !scores->score || n_req < 1 || L < 1) return RPS_ERR_INVALID_ARG;
@@ -268,17 +276,57 @@ rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L,
         !out->margin || !out->mask_pos || !out->mask_cnt)
         return RPS_ERR_INVALID_ARG;
     if (out->mask_pos == piv->rem_pos) return RPS_ERR_INVALID_ARG;
+    a->score = scores->score;
+    a->piv = *piv;
+    a->n_req = n_req;
+    a->L = L;
+    a->P = prm->n_pivots;
+    a->K = prm->tokens_per_pivot;
+    a->out = *out;
+    return RPS_OK;
+}
+
+}  // namespace
+}  // namespace rps
+
+extern "C" {
+
+rps_status rps_score_branches(const rps_logits *anchor_logits, int32_t anchor_branch,
+                              const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req,
+                              int32_t L, const rps_pivots *piv, const rps_params *prm,
+                              const rps_branch_scores *out, rps_stream_t stream) {
+    ScoreArgs a;
+    rps_status st = make_score_args(anchor_logits, anchor_branch, anchor, branch, n_req, L, piv, prm, out, &a);
+    if (st != RPS_OK) return st;
     DeviceInfo dev;
     if ((st = device_info(&dev)) != RPS_OK) return st;
+    a.err = dev.err;
+    return from_cuda(launch_score(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_commit(const rps_branch_scores *scores, int32_t n_req, int32_t L, const rps_pivots *piv,
+                      const rps_params *prm, const rps_commit_out *out, rps_stream_t stream) {
     CommitArgs a;
-    a.score = scores->score;
-    a.piv = *piv;
-    a.n_req = n_req;
-    a.L = L;
-    a.P = prm->n_pivots;
-    a.K = prm->tokens_per_pivot;
-    a.out = *out;
+    rps_status st = make_commit_args(scores, n_req, L, piv, prm, out, &a);
+    if (st != RPS_OK) return st;
+    DeviceInfo dev;
+    if ((st = device_info(&dev)) != RPS_OK) return st;
     return from_cuda(launch_commit(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_score_and_commit(const rps_logits *anchor_logits, int32_t anchor_branch,
+                                const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req, int32_t L,
+                                const rps_pivots *piv, const rps_params *prm, const rps_branch_scores *scores,
+                                const rps_commit_out *out, rps_stream_t stream) {
+    ScoreArgs s;
+    CommitArgs c;
+    rps_status st = make_score_args(anchor_logits, anchor_branch, anchor, branch, n_req, L, piv, prm, scores, &s);
+    if (st != RPS_OK) return st;
+    if ((st = make_commit_args(scores, n_req, L, piv, prm, out, &c)) != RPS_OK) return st;
+    DeviceInfo dev;
+    if ((st = device_info(&dev)) != RPS_OK) return st;
+    s.err = dev.err;
+    return from_cuda(launch_score_commit(s, c, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 rps_status rps_poll_device_status(rps_stream_t stream, uint32_t *detail) {

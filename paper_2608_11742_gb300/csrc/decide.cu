@@ -1,14 +1,17 @@
 // decide.cu -- per-request decision kernels of one RPS step.
 //
-//   select_kernel  standard commit (Eq. 2 with the fallback of Algorithm 1),
-//                  M' = M \ S, pivots (Eq. 3), candidate tokens (Sec. 3.1) and
-//                  the lookahead row list            -> rps_select_pivots
-//   score_kernel   Eq. 4 per (pivot, candidate) and N_tau (Proposition 1)
-//                                                    -> rps_score_branches
-//   commit_kernel  commit-or-abstain and the mask after the step
-//                                                    -> rps_commit
+//   select_kernel        standard commit (Eq. 2 with the fallback of Algorithm 1),
+//                        M' = M \ S, pivots (Eq. 3), candidate tokens (Sec. 3.1)
+//                        and the lookahead row list       -> rps_select_pivots
+//   score_kernel         Eq. 4 per (pivot, candidate) and N_tau (Proposition 1)
+//                                                         -> rps_score_branches
+//   commit_kernel        commit-or-abstain and the mask after the step
+//                                                         -> rps_commit
+//   score_commit_kernel  both of the above in one launch  -> rps_score_and_commit
 // One block per request; everything here is O(L * k) words, negligible next to
-// the row-statistics stream.
+// the row-statistics stream, so the kernels are written to keep dependent
+// global-memory round trips few: each block first stages what it needs in
+// shared memory with independent loads.
 #include <cfloat>
 #include <climits>
 
@@ -19,6 +22,7 @@ namespace {
 
 constexpr int kSelectThreads = 256;
 constexpr int kScoreThreads = 256;
+constexpr int kMaxSlots = RPS_MAX_PIVOTS * (RPS_MAX_K + 1);
 
 // Block-wide exclusive scan of one int per thread; returns the block total.
 __device__ __forceinline__ int block_excl_scan(int v, int &excl, int *warp_buf) {
@@ -41,7 +45,7 @@ __device__ __forceinline__ int block_excl_scan(int v, int &excl, int *warp_buf) 
     return total;
 }
 
-// Best entry of the block by (value desc, position asc); -1 when no thread has one.
+// Best entry of the block by (value desc, position asc); idx -1 when no thread has one.
 struct Best {
     float v;
     int pos;
@@ -73,6 +77,9 @@ __device__ Best block_best(Best mine, Best *buf) {
     return r;
 }
 
+// Dynamic shared memory of select_kernel per masked position.
+constexpr int kSelectBytesPerPos = 3 * sizeof(float) + 3 * sizeof(int32_t) + 2;
+
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs a) {
     const int q = blockIdx.x;
     const int tid = threadIdx.x;
@@ -82,10 +89,17 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
 
     __shared__ int warp_buf[kSelectThreads / 32];
     __shared__ Best best_buf[kSelectThreads / 32];
-    __shared__ uint8_t in_S[RPS_MAX_POS];
-    __shared__ uint8_t taken[RPS_MAX_POS];
-    __shared__ int piv_i[RPS_MAX_PIVOTS];   // index of pivot j in M'
+    __shared__ int piv_i[RPS_MAX_PIVOTS];  // index of pivot j in M'
     __shared__ int piv_nc[RPS_MAX_PIVOTS];
+    extern __shared__ __align__(16) unsigned char sel_smem[];
+    float *pm = reinterpret_cast<float *>(sel_smem);  // P^max of mask entry k
+    float *mu = pm + L;                                // retained mass
+    float *ht = mu + L;                                // truncated entropy
+    int32_t *pos = reinterpret_cast<int32_t *>(ht + L);  // position
+    int32_t *am = pos + L;                               // argmax token
+    int32_t *rk = am + L;                                // M' entry i -> mask entry
+    uint8_t *in_S = reinterpret_cast<uint8_t *>(rk + L);
+    uint8_t *taken = in_S + L;
 
     int cnt = a.mask_cnt[q];
     if (cnt < 0 || cnt > L) {
@@ -93,7 +107,14 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         cnt = cnt < 0 ? 0 : L;
     }
 
-    // Defaults for this request.
+    // Stage this request's statistics (independent loads) and write the defaults.
+    for (int k = tid; k < cnt; k += blockDim.x) {
+        pm[k] = a.pmax[base + k];
+        mu[k] = a.mu[base + k];
+        ht[k] = a.htrunc[base + k];
+        pos[k] = a.mask_pos[base + k];
+        am[k] = a.argmax[base + k];
+    }
     for (int j = tid; j < P; j += blockDim.x) {
         o.pivot_k[q * P + j] = -1;
         o.pivot_pos[q * P + j] = -1;
@@ -105,11 +126,12 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         o.branch_off[q * NB + b] = 0;
         o.branch_cnt[q * NB + b] = 0;
     }
+    __syncthreads();
 
     // Step 1: S = {i in M : P^max_i >= tau}; fallback to the most confident row.
     int any = 0;
     for (int k = tid; k < cnt; k += blockDim.x) {
-        const uint8_t f = a.pmax[base + k] >= a.tau;
+        const uint8_t f = pm[k] >= a.tau;
         in_S[k] = f;
         any |= f;
     }
@@ -117,7 +139,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
     if (!any && cnt > 0) {
         Best mine{-INFINITY, INT_MAX, -1};
         for (int k = tid; k < cnt; k += blockDim.x) {
-            Best c{a.pmax[base + k], a.mask_pos[base + k], k};
+            Best c{pm[k], pos[k], k};
             if (!(c.v == c.v)) c.v = -INFINITY;  // NaN statistics never win
             if (better(c, mine)) mine = c;
         }
@@ -134,14 +156,14 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         int excl;
         const int tot = block_excl_scan(f, excl, warp_buf);
         if (k < cnt) {
-            const int32_t pos = a.mask_pos[base + k];
             if (f) {
-                o.commit_pos[base + n_commit + excl] = pos;
-                o.commit_tok[base + n_commit + excl] = a.argmax[base + k];
+                o.commit_pos[base + n_commit + excl] = pos[k];
+                o.commit_tok[base + n_commit + excl] = am[k];
             } else {
                 const int r = k - (n_commit + excl);
+                rk[r] = k;
                 o.rem_k[base + r] = k;
-                o.rem_pos[base + r] = pos;
+                o.rem_pos[base + r] = pos[k];
             }
         }
         n_commit += tot;
@@ -156,18 +178,17 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         if (tid == 0) o.state[q] = RPS_STATE_DONE;
         return;
     }
-    __syncthreads();  // rem_k / rem_pos written above are read below
-
-    // Steps 3-4: feasibility (mu >= tau_pivot) and pivots by truncated entropy.
     for (int i = tid; i < n_rem; i += blockDim.x) taken[i] = 0;
     __syncthreads();
+
+    // Steps 3-4: feasibility (mu >= tau_pivot) and pivots by truncated entropy.
     int n_piv = 0;
     for (int j = 0; j < P; ++j) {
         Best mine{-INFINITY, INT_MAX, -1};
         for (int i = tid; i < n_rem; i += blockDim.x) {
-            const int k = o.rem_k[base + i];
-            if (taken[i] || !(a.mu[base + k] >= a.tau_pivot)) continue;
-            Best c{a.htrunc[base + k], o.rem_pos[base + i], i};
+            const int k = rk[i];
+            if (taken[i] || !(mu[k] >= a.tau_pivot)) continue;
+            Best c{ht[k], pos[k], i};
             if (!(c.v == c.v)) continue;
             if (better(c, mine)) mine = c;
         }
@@ -176,7 +197,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         if (tid == 0) {
             taken[b.idx] = 1;
             piv_i[j] = b.idx;
-            o.pivot_k[q * P + j] = o.rem_k[base + b.idx];
+            o.pivot_k[q * P + j] = rk[b.idx];
             o.pivot_pos[q * P + j] = b.pos;
         }
         n_piv = j + 1;
@@ -190,12 +211,13 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
     // Step 5: candidates z_v - zmax >= log r in rank order, at most K.
     if (tid < n_piv) {
         const int j = tid;
-        const int64_t row = base + o.rem_k[base + piv_i[j]];
+        const int64_t row = base + rk[piv_i[j]];
         const double zmax = a.zmax[row];
         int nc = 0;
         for (int t = 0; t < a.k_max && nc < K; ++t) {
             const double zt = a.topk_logit[row * a.k_max + t];
-            if (zt - zmax >= a.log_r) o.cand_tok[(static_cast<int64_t>(q) * P + j) * K + nc++] = a.topk_idx[row * a.k_max + t];
+            if (zt - zmax >= a.log_r)
+                o.cand_tok[(static_cast<int64_t>(q) * P + j) * K + nc++] = a.topk_idx[row * a.k_max + t];
         }
         piv_nc[j] = nc;
         o.n_cand[q * P + j] = nc;
@@ -229,7 +251,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
                     const int d = i < pi ? i : i - 1;
                     rows[d * 3 + 0] = q;
                     rows[d * 3 + 1] = 1 + b;
-                    rows[d * 3 + 2] = o.rem_pos[base + i];
+                    rows[d * 3 + 2] = pos[rk[i]];
                 }
             }
             off += n;
@@ -247,22 +269,39 @@ __device__ __forceinline__ float load_logit(const void *data, int dtype, int64_t
     return static_cast<const float *>(data)[e];
 }
 
-__global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a) {
-    const int q = blockIdx.x;
+// Pivot-selection facts of one request, staged in shared memory.
+struct PivotView {
+    int state, n_rem;
+    int pivot_k[RPS_MAX_PIVOTS];
+    int pivot_pos[RPS_MAX_PIVOTS];
+    int n_cand[RPS_MAX_PIVOTS];
+};
+
+__device__ void stage_pivots(const rps_pivots &pv, int q, int P, PivotView &v) {
+    if (threadIdx.x == 0) {
+        v.state = pv.state[q];
+        v.n_rem = pv.rem_cnt[q];
+    }
+    for (int j = threadIdx.x; j < P; j += blockDim.x) {
+        v.pivot_k[j] = pv.pivot_k[q * P + j];
+        v.pivot_pos[j] = pv.pivot_pos[q * P + j];
+        v.n_cand[j] = pv.n_cand[q * P + j];
+    }
+}
+
+// Eq. 4 scores of one request, one warp per (pivot, slot); also kept in `sc`.
+__device__ void score_request(const ScoreArgs &a, int q, const PivotView &v, float *sc) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
     const int L = a.L, P = a.P, K = a.K, NB = P * K;
     const int64_t base = static_cast<int64_t>(q) * L;
     const rps_pivots &pv = a.piv;
-    const int state = pv.state[q];
-    const int n_rem = pv.rem_cnt[q];
-
     for (int slot = w; slot < P * (K + 1); slot += nw) {
         const int j = slot / (K + 1), c = slot % (K + 1);
         const int64_t o = (static_cast<int64_t>(q) * P + j) * (K + 1) + c;
-        const int pk = pv.pivot_k[q * P + j];
+        const int pk = v.pivot_k[j];
         float mean_H = NAN, log_a = NAN, score = NAN;
         int n_tau = -1;
-        bool scored = state == RPS_STATE_SEARCH && pk >= 0 && pv.n_cand[q * P + j] >= 2;
+        bool scored = v.state == RPS_STATE_SEARCH && pk >= 0 && v.n_cand[j] >= 2;
         if (scored && c < K) scored = pv.branch_valid[q * NB + j * K + c] != 0;
         if (scored) {
             float sum = 0.f;
@@ -277,19 +316,19 @@ __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a)
                     count += a.b_pmax[first + i] >= a.tau;
                 }
                 const int tok = pv.cand_tok[(static_cast<int64_t>(q) * P + j) * K + c];
-                const int pos = pv.pivot_pos[q * P + j];
+                const int p = v.pivot_pos[j];
                 if (tok < 0 || tok >= a.vocab) {
                     if (lane == 0) flag_error(a.err, RPS_DEVERR_TOKEN);
                     la = NAN;
-                } else if (pos < 0 || pos >= a.n_pos) {
+                } else if (p < 0 || p >= a.n_pos) {
                     if (lane == 0) flag_error(a.err, RPS_DEVERR_ROW_INDEX);
                     la = NAN;
                 } else {
-                    const int64_t e = q * a.req_stride + a.branch_offset + pos * a.pos_stride + tok;
+                    const int64_t e = q * a.req_stride + a.branch_offset + p * a.pos_stride + tok;
                     la = load_logit(a.anchor_data, a.dtype, e) - a.a_lse[base + pk];
                 }
             } else {
-                for (int i = lane; i < n_rem; i += 32) {
+                for (int i = lane; i < v.n_rem; i += 32) {
                     const int k = pv.rem_k[base + i];
                     if (k == pk) continue;
                     sum += a.a_H[base + k];
@@ -299,7 +338,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a)
             }
             sum = warp_sum(sum);
             count = warp_sum_int(count);
-            const int n = n_rem - 1;
+            const int n = v.n_rem - 1;
             mean_H = n > 0 ? sum / static_cast<float>(n) : 0.f;
             n_tau = count;
             log_a = la;
@@ -310,13 +349,14 @@ __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a)
             a.out.n_tau[o] = n_tau;
             a.out.log_a[o] = log_a;
             a.out.score[o] = score;
+            if (sc) sc[slot] = score;
         }
     }
 }
 
-__global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
-    const int q = blockIdx.x;
-    const int lane = threadIdx.x;
+// Commit decision of one request by one warp; `s` holds the request's scores.
+__device__ void commit_request(const CommitArgs &a, int q, const float *s_req) {
+    const int lane = threadIdx.x & 31;
     const int L = a.L, P = a.P, K = a.K, NB = P * K;
     const int64_t base = static_cast<int64_t>(q) * L;
     const rps_pivots &pv = a.piv;
@@ -325,17 +365,17 @@ __global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
     // Best slot and gain of the pivot held by this lane.
     int best = -1;
     float gain = NAN;
-    int pos = INT_MAX;
+    int ppos = INT_MAX;
     bool wins = false;
     if (lane < P && state == RPS_STATE_SEARCH && pv.pivot_pos[q * P + lane] >= 0 && pv.n_cand[q * P + lane] >= 2) {
-        const float *s = a.score + (static_cast<int64_t>(q) * P + lane) * (K + 1);
+        const float *s = s_req + lane * (K + 1);
         best = K;
         for (int c = 0; c < K; ++c) {
             if (!pv.branch_valid[q * NB + lane * K + c]) continue;
             if (s[c] > s[best]) best = c;
         }
         gain = s[best] - s[K];
-        pos = pv.pivot_pos[q * P + lane];
+        ppos = pv.pivot_pos[q * P + lane];
         wins = best < K && gain > 0.f;
     }
     if (lane < P) {
@@ -344,7 +384,7 @@ __global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
     }
     // Pivot with the largest positive gain, lower position on ties.
     float g = wins ? gain : -INFINITY;
-    int p = wins ? pos : INT_MAX;
+    int p = wins ? ppos : INT_MAX;
     int j = wins ? lane : -1;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -392,10 +432,38 @@ __global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
     if (lane == 0) a.out.mask_cnt[q] = kept;
 }
 
+__global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a) {
+    __shared__ PivotView v;
+    stage_pivots(a.piv, blockIdx.x, a.P, v);
+    __syncthreads();
+    score_request(a, blockIdx.x, v, nullptr);
+}
+
+__global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
+    const int q = blockIdx.x;
+    commit_request(a, q, a.score + static_cast<int64_t>(q) * a.P * (a.K + 1));
+}
+
+__global__ void __launch_bounds__(kScoreThreads) score_commit_kernel(const ScoreArgs s, const CommitArgs c) {
+    __shared__ PivotView v;
+    __shared__ float sc[kMaxSlots];
+    stage_pivots(s.piv, blockIdx.x, s.P, v);
+    __syncthreads();
+    score_request(s, blockIdx.x, v, sc);
+    __syncthreads();
+    if (threadIdx.x < 32) commit_request(c, blockIdx.x, sc);
+}
+
 }  // namespace
 
 cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream) {
-    select_kernel<<<a.n_req, kSelectThreads, 0, stream>>>(a);
+    const size_t smem = static_cast<size_t>(a.L) * kSelectBytesPerPos + 16;
+    if (smem > 48 * 1024) {
+        const cudaError_t e =
+            cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+    }
+    select_kernel<<<a.n_req, kSelectThreads, smem, stream>>>(a);
     return cudaGetLastError();
 }
 
@@ -406,6 +474,11 @@ cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream) {
 
 cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream) {
     commit_kernel<<<a.n_req, 32, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStream_t stream) {
+    score_commit_kernel<<<s.n_req, kScoreThreads, 0, stream>>>(s, c);
     return cudaGetLastError();
 }
 

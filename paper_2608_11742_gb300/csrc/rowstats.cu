@@ -11,24 +11,34 @@
 // partial record in the workspace and the last warp to finish a row (atomic
 // ticket, no waiting) merges the at most kMaxPartials records and writes the row.
 //
+// Data movement. Each warp owns a ring of shared-memory buffers of 2 KB.
+// Lane 0 keeps every free buffer filled by a bulk asynchronous copy (cp.async.bulk, completion
+// counted on an mbarrier per buffer) in flight ahead of the warp, across row
+// boundaries; the lanes read their four 16-byte units of each buffer from shared
+// memory. Bytes in flight therefore cost no registers. Every mbarrier wait is
+// bounded: on expiry the warp flags RPS_DEVERR_TIMEOUT, waits (bounded) for its
+// own copies and stops.
+//
 // Per lane, a row segment is reduced as a base-2 online softmax against an
 // exponent reference mref that is raised only when a value exceeds it by more
-// than kSlack nats (rare), so the steady state is, per element, one FFMA, one
-// MUFU ex2 and two FP32 adds/FMAs:
+// than kSlack nats (rare):
 //   s = sum 2^u, t = sum u 2^u, u = (z - mref) log2(e)
 //   H = ln S - ln2 * T / S,  lse = mref + ln S   (after merging lanes / pieces)
-// The exact maximum is tracked per 16-byte unit; its token index is resolved
-// once per segment by re-reading the unit that holds it.
+// The exact maximum is tracked per unit; its token index is resolved once per
+// segment by re-reading the unit that holds it.
 //
-// Top-k (k <= 32) lives in a warp-distributed sorted list, lane j holding rank j
-// in the order (logit desc, token asc). Elements below a warp threshold are
-// discarded with one compare per unit; the threshold is the list's k-th value,
-// seeded after the first batch by the k-th largest lane maximum (a valid lower
-// bound: those k lanes each hold an element at least that large).
+// Top-k (k <= 32, top-k mode only) takes a sketch and a short second pass. While
+// streaming, each lane records its maximum over its units of every ring chunk
+// (one value per 64 bytes of logits) in the workspace. After the segment, the
+// k-th largest of the 32 lane maxima is a lower bound on the segment's k-th
+// largest logit (those k lanes each hold an element at least that large); only
+// the (chunk, lane) pairs whose recorded maximum reaches the bound -- a handful --
+// are reloaded from L2, and their elements at or above it enter a warp-
+// distributed sorted list (lane j holds rank j in the order logit desc, token asc).
 //
-// -inf logits or NaN make the fast path's t NaN; the segment is then rescanned
-// with clamped exponents (SAFE), which scores -inf as probability 0 and flags
-// NaN input as RPS_DEVERR_NONFINITE.
+// -inf logits or NaN make the first pass's sums NaN; the segment is then rescanned
+// from global memory with clamped exponents (SAFE), which scores -inf as
+// probability 0 and flags NaN input as RPS_DEVERR_NONFINITE.
 #include <cfloat>
 #include <climits>
 
@@ -39,8 +49,16 @@ namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr float kSlack = 8.0f;  // nats the reference may trail the maximum
+constexpr float kSlack = 8.0f;          // nats the reference may trail the maximum
+constexpr int kWarps = kRowThreads / 32;
+constexpr int kChunkUnits = 32 * kBatch;  // 16-byte units per ring buffer (2 KB)
+// Staging area of the top-k second pass (top-k mode only): a lane's units of one
+// chunk, then the round's candidates, kCandBatch (value, token) pairs at a time.
+constexpr int kStageUnits = 32 * kBatch;
+constexpr int kCandBatch = 32;
+constexpr uint64_t kWaitLimitNs = 200ull * 1000 * 1000;  // a bulk copy normally lands within microseconds
 
+// ---------------------------------------------------------------- PTX helpers
 __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -88,6 +106,73 @@ __device__ __forceinline__ uint4 ld_stream(const void *p) {
     return v;
 }
 
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Shared-memory 16-byte load the compiler may not merge with an earlier one (a
+// second read of a ring unit costs less than keeping the first in registers).
+__device__ __forceinline__ uint4 lds_again(const uint4 *p) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(smem_u32(p)));
+    return v;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+
+// Orders this thread's earlier shared-memory accesses before later async-proxy writes.
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Arm `bar` for `bytes` and start a bulk copy of them from global memory into `dst`.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Waits for phase `parity` of `bar`, giving up after kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t start = global_ns();
+    while (global_ns() - start < kWaitLimitNs)
+        if (mbar_try_wait(bar, parity)) return true;
+    return false;
+}
+
+__device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+// ---------------------------------------------------------------- element types
 template <int DT>
 struct Elem;
 
@@ -104,6 +189,23 @@ struct Elem<RPS_BF16> {
         y[5] = __uint_as_float(w.z & 0xffff0000u);
         y[6] = __uint_as_float(w.w << 16);
         y[7] = __uint_as_float(w.w & 0xffff0000u);
+    }
+    __device__ static __forceinline__ float unit_max(const uint4 &w) {
+        const uint32_t m = bf16x2_max(bf16x2_max(w.x, w.y), bf16x2_max(w.z, w.w));
+        return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
+    }
+    // per-(chunk, lane) maximum kept for the top-k second pass: the bf16 bits
+    typedef uint16_t Sketch;
+    __device__ static __forceinline__ Sketch to_sketch(float v) { return static_cast<uint16_t>(__float_as_uint(v) >> 16); }
+    __device__ static __forceinline__ float from_sketch(Sketch s) { return __uint_as_float(static_cast<uint32_t>(s) << 16); }
+    // running maximum of whole units, kept as a packed bf16 pair
+    typedef uint32_t Acc;
+    __device__ static __forceinline__ Acc acc_init() { return 0xff80ff80u; }  // (-inf, -inf)
+    __device__ static __forceinline__ Acc acc_add(Acc m, const uint4 &w) {
+        return bf16x2_max(bf16x2_max(m, w.x), bf16x2_max(bf16x2_max(w.y, w.z), w.w));
+    }
+    __device__ static __forceinline__ float acc_value(Acc m) {
+        return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xffff0000u));
     }
     __device__ static __forceinline__ float load1(const char *row, int64_t e) {
         return __uint_as_float(static_cast<uint32_t>(reinterpret_cast<const uint16_t *>(row)[e]) << 16);
@@ -125,20 +227,35 @@ struct Elem<RPS_F32> {
         y[2] = __uint_as_float(w.z);
         y[3] = __uint_as_float(w.w);
     }
+    __device__ static __forceinline__ float unit_max(const uint4 &w) {
+        return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)), fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+    }
+    typedef float Sketch;
+    __device__ static __forceinline__ Sketch to_sketch(float v) { return v; }
+    __device__ static __forceinline__ float from_sketch(Sketch s) { return s; }
+    typedef float Acc;
+    __device__ static __forceinline__ Acc acc_init() { return -INFINITY; }
+    __device__ static __forceinline__ Acc acc_add(Acc m, const uint4 &w) { return fmaxf(m, unit_max(w)); }
+    __device__ static __forceinline__ float acc_value(Acc m) { return m; }
     __device__ static __forceinline__ float load1(const char *row, int64_t e) {
         return reinterpret_cast<const float *>(row)[e];
     }
-    __device__ static __forceinline__ float pick(const uint32_t *words, int i) {
-        return __uint_as_float(words[i]);
-    }
+    __device__ static __forceinline__ float pick(const uint32_t *words, int i) { return __uint_as_float(words[i]); }
 };
 
+// True when this lane holds at least one unit of a chunk of n_units units.
+__device__ __forceinline__ bool j0_valid(int n_units, int lane) { return lane < n_units; }
+
+// ---------------------------------------------------------------- online softmax
 struct LaneState {
-    float mref;   // exponent reference, -inf until the first finite value
-    f2 s, t;      // pairwise partial sums of 2^u and u 2^u, u = (z - mref) log2(e)
-    float mx;     // exact running maximum
-    int best;     // first element of the unit where mx was first reached, -1 if none
-    bool bad;     // NaN input seen (SAFE scan only)
+    float mref;       // exponent reference, -inf until the first finite value
+    f2 s, t;          // pairwise partial sums of 2^u and u 2^u, u = (z - mref) log2(e)
+    float mx;         // exact running maximum
+    int best;         // unit (or first unit of the ring chunk) where mx was first reached, -1 if none
+    bool best_chunk;  // best names a ring chunk: this lane's units best + 32 j, j < kBatch
+    bool bad;         // NaN input seen (SAFE scan only)
+    float c1v, c2v;   // top-k mode: this lane's two largest chunk maxima ...
+    int c1u, c2u;     // ... and the first units of those chunks (-1 if none)
 };
 
 __device__ __forceinline__ void lane_init(LaneState &L) {
@@ -147,34 +264,33 @@ __device__ __forceinline__ void lane_init(LaneState &L) {
     L.t = pack2(0.f, 0.f);
     L.mx = -INFINITY;
     L.best = -1;
+    L.best_chunk = false;
     L.bad = false;
+    L.c1v = L.c2v = -INFINITY;
+    L.c1u = L.c2u = -1;
 }
 
-// Fold one unit of n valid values (n == N except for a ragged row tail). The
-// exponent is formed as (z - mref) * log2(e): the difference is exact for
-// values near the reference, so large logits lose no absolute precision.
-template <int N, bool SAFE>
-__device__ __forceinline__ float fold_unit(LaneState &L, const float (&y)[N], int n, int e0) {
-    float vmax = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < N; ++i)
-        if (i < n) vmax = fmaxf(vmax, y[i]);
-    if (vmax > L.mx) {
-        L.mx = vmax;
-        L.best = e0;
-    }
-    if (vmax > L.mref + kSlack) {  // raise the exponent reference (rare)
+// Raise the exponent reference to m (rare: only when m exceeds it by kSlack).
+__device__ __forceinline__ void raise_reference(LaneState &L, float m) {
+    if (m > L.mref + kSlack) {
         float slo, shi;
         unpack2(L.s, slo, shi);
         if (slo + shi > 0.f) {
-            const float d = (L.mref - vmax) * kLog2e;
+            const float d = (L.mref - m) * kLog2e;
             const float a = ex2(d);
             const f2 a2 = pack2(a, a);
             L.t = mul2(a2, fma2(pack2(d, d), L.s, L.t));
             L.s = mul2(a2, L.s);
         }
-        L.mref = vmax;
+        L.mref = m;
     }
+}
+
+// Sums of n values (n even or the last value alone). The exponent is formed as
+// (z - mref) * log2(e): the difference is exact for values near the reference,
+// so large logits lose no absolute precision.
+template <int N, bool SAFE>
+__device__ __forceinline__ void accumulate(LaneState &L, const float (&y)[N], int n) {
     const f2 m2 = pack2(L.mref, L.mref);
     const f2 l2 = pack2(kLog2e, kLog2e);
 #pragma unroll
@@ -196,9 +312,106 @@ __device__ __forceinline__ float fold_unit(LaneState &L, const float (&y)[N], in
         L.s = add2(L.s, e2);
         L.t = fma2(uu, e2, L.t);
     }
-    return vmax;
 }
 
+// Fold one unit of n valid values (n == N except for a ragged row tail).
+template <int N, bool SAFE>
+__device__ __forceinline__ void fold_unit(LaneState &L, const float (&y)[N], int n, int unit) {
+    float vmax = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < N; ++i)
+        if (i < n) vmax = fmaxf(vmax, y[i]);
+    if (vmax > L.mx) {
+        L.mx = vmax;
+        L.best = unit;
+        L.best_chunk = false;
+    }
+    raise_reference(L, vmax);
+    accumulate<N, SAFE>(L, y, n);
+}
+
+// Fold this lane's units of one ring chunk (the fast path). The chunk's maximum
+// comes from packed compares; the exact argmax is resolved once per segment.
+template <int DT, bool TOPK>
+__device__ __forceinline__ float fold_chunk(LaneState &L, typename Elem<DT>::Sketch *sketch, const uint4 *buf,
+                                            int n_units, int cu, int lane) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    typename E::Acc acc = E::acc_init();
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j)
+        if (j * 32 + lane < n_units) acc = E::acc_add(acc, buf[j * 32 + lane]);
+    const float cmax = j0_valid(n_units, lane) ? E::acc_value(acc) : -INFINITY;
+    if (cmax > L.mx) {
+        L.mx = cmax;
+        L.best = cu;
+        L.best_chunk = true;
+    }
+    raise_reference(L, cmax);
+    if (TOPK && j0_valid(n_units, lane)) {
+        sketch[cu + lane] = E::to_sketch(cmax);
+        if (cmax > L.c2v) {  // keep the two largest chunk maxima
+            if (cmax > L.c1v) {
+                L.c2v = L.c1v;
+                L.c2u = L.c1u;
+                L.c1v = cmax;
+                L.c1u = cu;
+            } else {
+                L.c2v = cmax;
+                L.c2u = cu;
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+        if (j * 32 + lane < n_units) {
+            float y[N];
+            E::unpack(lds_again(buf + j * 32 + lane), y);
+            accumulate<N, false>(L, y, N);
+        }
+    }
+    return cmax;
+}
+
+// The ragged last unit of a row (fewer than N values), folded by lane 0.
+template <int DT, bool SAFE>
+__device__ __forceinline__ void fold_tail(LaneState &L, const char *row, int V, int lane) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    const int e0 = (V / N) * N;
+    const int n = V - e0;
+    if (lane != 0 || n == 0) return;
+    float y[N];
+#pragma unroll
+    for (int i = 0; i < N; ++i) y[i] = i < n ? E::load1(row, e0 + i) : -INFINITY;
+    fold_unit<N, SAFE>(L, y, n, V / N);
+}
+
+// Rescan of a segment straight from global memory with clamped exponents; used
+// when the fast pass saw -inf or NaN.
+template <int DT>
+__device__ void rescan_safe(LaneState &L, const char *row, int V, int u0, int u1, int lane) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    // the top-k chunk record of the fast pass stays valid: -inf and NaN do not
+    // change a chunk's maximum
+    const float c1v = L.c1v, c2v = L.c2v;
+    const int c1u = L.c1u, c2u = L.c2u;
+    lane_init(L);
+    L.c1v = c1v;
+    L.c2v = c2v;
+    L.c1u = c1u;
+    L.c2u = c2u;
+    const int full_end = min(u1, V / N);
+    for (int u = u0 + lane; u < full_end; u += 32) {
+        float y[N];
+        E::unpack(ld_stream(row + static_cast<size_t>(u) * 16), y);
+        fold_unit<N, true>(L, y, N, u);
+    }
+    if (u1 > V / N) fold_tail<DT, true>(L, row, V, lane);
+}
+
+// ---------------------------------------------------------------- top-k
 // True when (av, ai) ranks before (bv, bi): larger logit, then lower token id.
 __device__ __forceinline__ bool ranks_before(float av, int ai, float bv, int bi) {
     return av > bv || (av == bv && ai < bi);
@@ -234,128 +447,186 @@ __device__ __forceinline__ float warp_kth_largest(float x, int k, int lane) {
     return __shfl_sync(kFull, x, k - 1);
 }
 
-template <int DT, bool TOPK, bool SAFE>
-__device__ __forceinline__ void scan_segment(const char *row, int V, int u0, int u1, int k, int lane,
-                                             LaneState &L, float &tv, int &ti, uint4 *stage) {
+// Merges one candidate per lane (sentinel -inf / INT_MAX for none) into the
+// warp-distributed sorted list: bitonic sort of the 32 candidates in rank order,
+// then the element-wise better of the list and the reversed candidates (the 32
+// best of both, as a bitonic sequence), then a bitonic merge. Fixed cost,
+// independent of how many candidates are real.
+__device__ __forceinline__ void pair_step(float &v, int &i, int stride, bool keep_better) {
+    const float ov = __shfl_xor_sync(kFull, v, stride);
+    const int oi = __shfl_xor_sync(kFull, i, stride);
+    if (keep_better == ranks_before(ov, oi, v, i)) {
+        v = ov;
+        i = oi;
+    }
+}
+
+__device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, int ci, int k, int lane) {
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1)
+            pair_step(cv, ci, stride, ((lane & size) == 0) == ((lane & stride) == 0));
+    }
+    const float rv = __shfl_sync(kFull, cv, 31 - lane);
+    const int ri = __shfl_sync(kFull, ci, 31 - lane);
+    if (ranks_before(rv, ri, tv, ti)) {
+        tv = rv;
+        ti = ri;
+    }
+#pragma unroll
+    for (int stride = 16; stride > 0; stride >>= 1) pair_step(tv, ti, stride, (lane & stride) == 0);
+    if (lane >= k) {
+        tv = -INFINITY;
+        ti = INT_MAX;
+    }
+}
+
+// Second pass of a segment (top-k mode). theta is a lower bound on the segment's
+// k-th largest logit, so only the (chunk, lane) pairs whose recorded maximum
+// reaches it can hold a member of the top k. Each lane loads kGroup of its
+// recorded maxima at once and marks its hits; then, round after round, every lane
+// with a hit left reloads that chunk's units (from L2) at the same time, and the
+// warp merges their elements at or above max(theta, current k-th entry) into the
+// warp-distributed list, 32 at a time (warp_merge_batch).
+template <int DT>
+__device__ __forceinline__ void topk_round(const char *row, int cend, int cu, int k, int lane, float theta, float &tv,
+                                           int &ti, uint4 *stage, float2 *cand) {
     using E = Elem<DT>;
     constexpr int N = E::N;
-    lane_init(L);
+    static_assert(kBatch * N <= 64, "candidate mask holds 64 elements");
+    const uint32_t *words = reinterpret_cast<const uint32_t *>(stage);
+    const float th = fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
+    unsigned long long cm = 0;
+    if (cu >= 0) {
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int u = cu + j * 32 + lane;
+            if (u < cend) {
+                const uint4 w = ld_stream(row + static_cast<size_t>(u) * 16);
+                stage[lane * kBatch + j] = w;
+                float y[N];
+                E::unpack(w, y);
+#pragma unroll
+                for (int i = 0; i < N; ++i)
+                    if (y[i] >= th) cm |= 1ull << (j * N + i);
+            }
+        }
+    }
+    // compact the round's candidates into the candidate buffer, then merge
+    const int c = __popc(static_cast<unsigned>(cm)) + __popc(static_cast<unsigned>(cm >> 32));
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += n;
+    }
+    const int total = __shfl_sync(kFull, incl, 31);
+    __syncwarp();
+    for (int done = 0; done < total; done += kCandBatch) {
+        // lanes write the candidates that fall in [done, done + kCandBatch)
+        int slot = incl - c;
+        unsigned long long bits = cm;
+        while (bits) {
+            const int bit = __ffsll(static_cast<long long>(bits)) - 1;
+            bits &= bits - 1;
+            if (slot >= done && slot < done + kCandBatch) {
+                const int j = bit / N, i = bit % N;
+                cand[slot - done] = make_float2(E::pick(words + (lane * kBatch + j) * 4, i),
+                                                __int_as_float((cu + j * 32 + lane) * N + i));
+            }
+            ++slot;
+        }
+        __syncwarp();
+        const int idx = done + lane;
+        const float2 e = idx < total ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
+        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane);
+        __syncwarp();
+    }
+}
+
+template <int DT>
+__device__ void topk_from_sketch(const LaneState &L, const char *row, const typename Elem<DT>::Sketch *sketch, int u0,
+                                 int cend, int k, int lane, float theta, float &tv, int &ti, uint4 *stage,
+                                 float2 *cand) {
+    using E = Elem<DT>;
+    constexpr int kGroup = 16;  // recorded maxima a lane loads together
     tv = -INFINITY;
     ti = INT_MAX;
-    float seed = -INFINITY;  // lower bound on the segment's k-th largest value
-    const int full_end = min(u1, V / N);  // units wholly inside the row
-    constexpr int step = 32 * kBatch;
-    bool first = true;
-
-    uint4 cur[kBatch];
+    // Usually a lane's only chunks at or above the bound are its two best.
+    topk_round<DT>(row, cend, L.c1v >= theta ? L.c1u : -1, k, lane, theta, tv, ti, stage, cand);
+    if (__any_sync(kFull, L.c2v >= theta))
+        topk_round<DT>(row, cend, L.c2v >= theta ? L.c2u : -1, k, lane, theta, tv, ti, stage, cand);
+    // A lane whose second best chunk reaches the bound may have more: scan its
+    // recorded maxima for the rest.
+    const bool more = L.c2v >= theta;
+    if (!__any_sync(kFull, more)) return;
+    for (int c0 = u0; c0 < cend; c0 += kGroup * kChunkUnits) {
+        float m[kGroup];
 #pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-        const int u = u0 + j * 32 + lane;
-        if (u < full_end) cur[j] = ld_stream(row + static_cast<size_t>(u) * 16);
-    }
-    for (int b = u0; b < full_end; b += step) {
-        uint4 nxt[kBatch];
-#pragma unroll
-        for (int j = 0; j < kBatch; ++j) {
-            const int u = b + step + j * 32 + lane;
-            if (u < full_end) nxt[j] = ld_stream(row + static_cast<size_t>(u) * 16);
+        for (int g = 0; g < kGroup; ++g) {
+            const int key = c0 + g * kChunkUnits + lane;
+            m[g] = more && key < cend ? E::from_sketch(sketch[key]) : -INFINITY;
         }
-        float bmax = -INFINITY;
+        const float th0 = fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
+        uint32_t hits = 0;
 #pragma unroll
-        for (int j = 0; j < kBatch; ++j) {
-            const int u = b + j * 32 + lane;
-            if (u < full_end) {
-                float y[N];
-                E::unpack(cur[j], y);
-                bmax = fmaxf(bmax, fold_unit<N, SAFE>(L, y, N, u * N));
-            }
+        for (int g = 0; g < kGroup; ++g) {
+            const int cu = c0 + g * kChunkUnits;
+            if (m[g] >= th0 && cu != L.c1u && cu != L.c2u) hits |= 1u << g;
         }
-        if (TOPK) {
-            if (first) {
-                seed = warp_kth_largest(bmax, k, lane);
-                first = false;
+        while (__any_sync(kFull, hits != 0)) {
+            int cu = -1;
+            if (hits) {
+                cu = c0 + (__ffs(hits) - 1) * kChunkUnits;
+                hits &= hits - 1;
             }
-            float th = fmaxf(__shfl_sync(kFull, tv, k - 1), seed);
-            if (__any_sync(kFull, bmax >= th)) {
-                // stage this batch and extract its candidates one at a time
-                unsigned cm = 0;
-#pragma unroll
-                for (int j = 0; j < kBatch; ++j) {
-                    const int u = b + j * 32 + lane;
-                    if (u < full_end) {
-                        stage[lane * kBatch + j] = cur[j];
-                        float y[N];
-                        E::unpack(cur[j], y);
-#pragma unroll
-                        for (int i = 0; i < N; ++i)
-                            if (y[i] >= th) cm |= 1u << (j * N + i);
-                    }
-                }
-                __syncwarp();
-                const uint32_t *words = reinterpret_cast<const uint32_t *>(stage);
-                while (true) {
-                    const unsigned lanes = __ballot_sync(kFull, cm != 0);
-                    if (!lanes) break;
-                    const int src = __ffs(lanes) - 1;
-                    const int bit = __shfl_sync(kFull, __ffs(cm) - 1, src);
-                    if (lane == src) cm &= cm - 1;
-                    const int j = bit / N, i = bit % N;
-                    const float cv = E::pick(words + (src * kBatch + j) * 4, i);
-                    if (cv >= th) {
-                        const int ci = (b + j * 32 + src) * N + i;
-                        topk_insert(tv, ti, cv, ci, k, lane);
-                        th = fmaxf(__shfl_sync(kFull, tv, k - 1), seed);
-                    }
-                }
-                __syncwarp();
-            }
-        }
-#pragma unroll
-        for (int j = 0; j < kBatch; ++j) cur[j] = nxt[j];
-    }
-
-    // ragged tail: the last unit of the row holds fewer than N values
-    if (u1 > full_end && full_end == V / N) {
-        const int e0 = full_end * N;
-        const int n = V - e0;
-        float y[N];
-#pragma unroll
-        for (int i = 0; i < N; ++i) y[i] = (i < n && lane == 0) ? E::load1(row, e0 + i) : -INFINITY;
-        float tmax = -INFINITY;
-        if (lane == 0) tmax = fold_unit<N, SAFE>(L, y, n, e0);
-        if (TOPK) {
-            if (first) seed = warp_kth_largest(tmax, k, lane);
-            float th = fmaxf(__shfl_sync(kFull, tv, k - 1), seed);
-#pragma unroll
-            for (int i = 0; i < N; ++i) {
-                const float cv = __shfl_sync(kFull, y[i], 0);
-                if (i < n && cv >= th) {
-                    topk_insert(tv, ti, cv, e0 + i, k, lane);
-                    th = fmaxf(__shfl_sync(kFull, tv, k - 1), seed);
-                }
-            }
+            topk_round<DT>(row, cend, cu, k, lane, theta, tv, ti, stage, cand);
         }
     }
 }
 
-// Lowest token index holding value mx among this lane's best unit (INT_MAX if none).
+// Candidates of a row's ragged last unit (top-k mode).
 template <int DT>
-__device__ __forceinline__ int resolve_argmax(const char *row, int64_t V, const LaneState &L, float MX) {
+__device__ __forceinline__ void topk_tail(const char *row, int V, int k, int lane, float &tv, int &ti) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    const int e0 = (V / N) * N;
+    const int n = V - e0;
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const float cv = i < n ? E::load1(row, e0 + i) : -INFINITY;
+        const float th = __shfl_sync(kFull, tv, k - 1);
+        if (i < n && cv >= th) topk_insert(tv, ti, cv, e0 + i, k, lane);
+    }
+}
+
+// ---------------------------------------------------------------- row records
+// Lowest token index holding value MX among the units this lane recorded as best
+// (INT_MAX if none).
+template <int DT>
+__device__ __forceinline__ int resolve_argmax(const char *row, int V, const LaneState &L, float MX, int lane) {
     using E = Elem<DT>;
     constexpr int N = E::N;
     if (L.best < 0 || !(L.mx == MX)) return INT_MAX;
-    const int64_t e0 = L.best;
-    const int n = static_cast<int>((V - e0 < N ? V - e0 : static_cast<int64_t>(N)));
-    float y[N];
-    if (n == N) {
-        E::unpack(ld_stream(row + e0 * E::kBytes), y);
-    } else {
+    const int full_units = V / N;
+    const int n_units = L.best_chunk ? kBatch : 1;
+    for (int j = 0; j < n_units; ++j) {
+        const int u = L.best_chunk ? L.best + j * 32 + lane : L.best;
+        const int e0 = u * N;
+        const int n = u < full_units ? N : V - e0;
+        if (n <= 0) break;
+        float y[N];
+        if (n == N) {
+            E::unpack(ld_stream(row + static_cast<size_t>(e0) * E::kBytes), y);
+        } else {
 #pragma unroll
-        for (int i = 0; i < N; ++i) y[i] = i < n ? E::load1(row, e0 + i) : -INFINITY;
+            for (int i = 0; i < N; ++i) y[i] = i < n ? E::load1(row, e0 + i) : -INFINITY;
+        }
+#pragma unroll
+        for (int i = 0; i < N; ++i)
+            if (i < n && y[i] == MX) return e0 + i;
     }
-#pragma unroll
-    for (int i = 0; i < N; ++i)
-        if (i < n && y[i] == MX) return static_cast<int>(e0 + i);
     return INT_MAX;
 }
 
@@ -423,20 +694,140 @@ __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, c
     }
 }
 
+// Merge of the top-k lists of every piece of a row (last arriver only), 32
+// entries per batch.
+__device__ __forceinline__ void merge_topk(const float2 *lists, int count, int k, int lane, float &tv, int &ti) {
+    const float2 e = __ldcg(lists + lane % k);  // list 0 seeds the merged list
+    tv = lane < k ? e.x : -INFINITY;
+    ti = lane < k ? __float_as_int(e.y) : INT_MAX;
+    const int total = count * k;
+    constexpr int kPer = 4;  // batches whose entries are loaded together
+    for (int base = k; base < total; base += 32 * kPer) {
+        float2 f[kPer];
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+            const int idx = base + q * 32 + lane;
+            f[q] = idx < total ? __ldcg(lists + idx) : make_float2(-INFINITY, __int_as_float(INT_MAX));
+        }
+#pragma unroll
+        for (int q = 0; q < kPer; ++q)
+            if (base + q * 32 < total) warp_merge_batch(tv, ti, f[q].x, __float_as_int(f[q].y), k, lane);
+    }
+}
+
+// ---------------------------------------------------------------- segments
+struct Segment {
+    int64_t slot;
+    const char *row;
+    int u0, u1;   // row-local unit range of this piece
+    bool valid;   // false: skipped entry or bad descriptor
+    bool bad;     // bad descriptor (to flag)
+};
+
+// Row r of the concatenated list -> (segment, entry) -> output slot and row pointer.
+template <int DT>
+__device__ __forceinline__ void locate(const RowStatsArgs &a, const int32_t *seg_start, int64_t r, Segment &s) {
+    int seg;
+    if (a.seg_cnt) {
+        int lo = 0, hi = a.n_seg;  // s with seg_start[s] <= r < seg_start[s + 1]
+        while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (seg_start[mid] <= r) lo = mid;
+            else hi = mid;
+        }
+        seg = lo;
+        s.slot = static_cast<int64_t>(lo) * a.cap + (r - seg_start[lo]);
+    } else {
+        seg = static_cast<int>(r / a.cap);
+        s.slot = r;
+    }
+    int32_t req, br, pos;
+    if (a.rows) {
+        req = a.rows[s.slot * 3 + 0];
+        br = a.rows[s.slot * 3 + 1];
+        pos = a.rows[s.slot * 3 + 2];
+    } else {
+        req = seg;
+        br = a.mask_branch;
+        pos = a.mask_pos[s.slot];
+    }
+    s.bad = pos >= 0 && (req < 0 || req >= a.n_req || br < 0 || br >= a.n_branch || pos >= a.n_pos);
+    s.valid = pos >= 0 && !s.bad;
+    s.row = s.valid ? static_cast<const char *>(a.data) +
+                          (req * a.req_stride + br * a.branch_stride + static_cast<int64_t>(pos) * a.pos_stride) *
+                              Elem<DT>::kBytes
+                    : nullptr;
+}
+
+// Walks the row segments of the global unit range [g, g_end).
+template <int DT>
+__device__ __forceinline__ bool next_segment(const RowStatsArgs &a, const int32_t *seg_start, int64_t nv, int64_t &g,
+                                             int64_t g_end, int64_t &r, Segment &s) {
+    if (g >= g_end) return false;
+    r = g / nv;
+    s.u0 = static_cast<int>(g - r * nv);
+    s.u1 = static_cast<int>(min(nv, static_cast<int64_t>(s.u0) + (g_end - g)));
+    g += s.u1 - s.u0;
+    locate<DT>(a, seg_start, r, s);
+    return true;
+}
+
+// Lane 0's copy engine: the next run of at most kChunkUnits whole units of the
+// piece, in the order the warp consumes them (valid segments only).
+template <int DT>
+struct Producer {
+    int64_t g, g_end;
+    Segment s;
+    int cu;      // next unit to copy in the current segment
+    int cu_end;  // end of its whole units
+    bool have;
+
+    __device__ __forceinline__ void init(int64_t g0, int64_t g1) {
+        g = g0;
+        g_end = g1;
+        have = false;
+        cu = cu_end = 0;
+    }
+
+    __device__ __forceinline__ bool next(const RowStatsArgs &a, const int32_t *seg_start, int64_t nv, int full_units,
+                                         const char *&src, uint32_t &bytes) {
+        while (!have || cu >= cu_end) {
+            int64_t r;
+            if (!next_segment<DT>(a, seg_start, nv, g, g_end, r, s)) return false;
+            have = s.valid;
+            cu = s.u0;
+            cu_end = min(s.u1, full_units);
+        }
+        const int n = min(kChunkUnits, cu_end - cu);
+        src = s.row + static_cast<size_t>(cu) * 16;
+        bytes = static_cast<uint32_t>(n) * 16u;
+        cu += n;
+        return true;
+    }
+};
+
 template <int DT, bool TOPK>
-__global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) row_stats_kernel(const RowStatsArgs a) {
+__global__ void __launch_bounds__(kRowThreads, 4) row_stats_kernel(const RowStatsArgs a) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    extern __shared__ __align__(128) uint4 dyn[];
     __shared__ int32_t seg_start[RPS_MAX_SEGMENTS + 1];
-    __shared__ uint4 stage_all[TOPK ? (kRowThreads / 32) * 32 * kBatch : 1];
+    __shared__ int32_t warp_total[kWarps];
+    constexpr int kRing = kStages;
+    __shared__ __align__(8) uint64_t bars[kWarps][kRing];
+
     const int lane = threadIdx.x & 31;
-    const int warp_in_block = threadIdx.x >> 5;
-    const int warp = blockIdx.x * (kRowThreads / 32) + warp_in_block;
-    uint4 *stage = stage_all + (TOPK ? warp_in_block * 32 * kBatch : 0);
+    const int wib = threadIdx.x >> 5;
+    const int warp = blockIdx.x * kWarps + wib;
+    uint4 *ring = dyn + wib * (kRing * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0));
+    uint4 *stage = ring + kRing * kChunkUnits;  // top-k candidate staging (top-k mode only)
+    float2 *cand = reinterpret_cast<float2 *>(stage + kStageUnits);
+    uint64_t *bar = bars[wib];
 
     // Exclusive prefix of the segment counts (clamped to capacity), four
     // segments per thread, then a block-wide scan.
     int64_t total_rows;
     if (a.seg_cnt) {
-        __shared__ int32_t warp_total[kRowThreads / 32];
         constexpr int kPer = RPS_MAX_SEGMENTS / kRowThreads;
         int32_t c[kPer];
         int32_t local = 0;
@@ -457,10 +848,10 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) row_stats_kernel(c
             const int32_t n = __shfl_up_sync(kFull, incl, o);
             if (lane >= o) incl += n;
         }
-        if (lane == 31) warp_total[warp_in_block] = incl;
+        if (lane == 31) warp_total[wib] = incl;
         __syncthreads();
         int32_t run = incl - local;
-        for (int w = 0; w < warp_in_block; ++w) run += warp_total[w];
+        for (int w = 0; w < wib; ++w) run += warp_total[w];
 #pragma unroll
         for (int i = 0; i < kPer; ++i) {
             seg_start[threadIdx.x * kPer + i] = run;
@@ -480,65 +871,100 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) row_stats_kernel(c
     const int64_t g_begin = static_cast<int64_t>(warp) * piece;
     if (g_begin >= total) return;
     const int64_t g_end = min(g_begin + piece, total);
-    const char *base = static_cast<const char *>(a.data);
-    constexpr int kBytes = Elem<DT>::kBytes;
+    const int V = static_cast<int>(a.vocab);
+    const int full_units = V / N;
 
-    for (int64_t g = g_begin; g < g_end;) {
-        const int64_t r = g / nv;
-        const int64_t u0 = g - r * nv;
-        const int64_t u1 = min(nv, u0 + (g_end - g));
-        g += u1 - u0;
+    // Ring set-up: one mbarrier per buffer, then up to kRing copies in flight.
+    if (lane == 0) {
+        for (int i = 0; i < kRing; ++i) mbar_init(bar + i, 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    Producer<DT> prod;
+    prod.init(g_begin, g_end);
+    int issued = 0;
+    if (lane == 0) {
+        const char *src;
+        uint32_t bytes;
+        while (issued < kRing && prod.next(a, seg_start, nv, full_units, src, bytes)) {
+            bulk_load(ring + issued * kChunkUnits, src, bytes, bar + issued);
+            ++issued;
+        }
+    }
+    issued = __shfl_sync(kFull, issued, 0);
+    int acquired = 0, released = 0;
 
-        // row r of the concatenated list -> (segment, entry) -> slot
-        int64_t slot;
-        int seg;
-        if (a.seg_cnt) {
-            int lo = 0, hi = a.n_seg;  // find s with seg_start[s] <= r < seg_start[s + 1]
-            while (hi - lo > 1) {
-                const int mid = (lo + hi) >> 1;
-                if (seg_start[mid] <= r) lo = mid; else hi = mid;
+    // Waits for the next ring chunk; false when the copy never lands (then this
+    // warp has flagged the error and drained its other copies: it must stop).
+    auto acquire = [&](int &st) -> bool {
+        st = acquired % kRing;
+        if (mbar_wait_bounded(bar + st, (acquired / kRing) & 1)) {
+            ++acquired;
+            return true;
+        }
+        if (lane == 0) {
+            flag_error(a.err, RPS_DEVERR_TIMEOUT);
+            for (int c = acquired + 1; c < issued; ++c) mbar_wait_bounded(bar + (c % kRing), (c / kRing) & 1);
+        }
+        __syncwarp();
+        return false;
+    };
+    // Hands the oldest held buffer back to the copy engine, which refills it.
+    auto release = [&]() {
+        const int st = released % kRing;
+        fence_proxy_async();
+        __syncwarp();
+        ++released;
+        if (lane == 0) {
+            const char *src;
+            uint32_t bytes;
+            if (prod.next(a, seg_start, nv, full_units, src, bytes)) {
+                bulk_load(ring + st * kChunkUnits, src, bytes, bar + st);
+                ++issued;
             }
-            seg = lo;
-            slot = static_cast<int64_t>(lo) * a.cap + (r - seg_start[lo]);
-        } else {
-            seg = static_cast<int>(r / a.cap);
-            slot = r;
         }
-        int32_t req, br, pos;
-        if (a.rows) {
-            req = a.rows[slot * 3 + 0];
-            br = a.rows[slot * 3 + 1];
-            pos = a.rows[slot * 3 + 2];
-        } else {
-            req = seg;
-            br = a.mask_branch;
-            pos = a.mask_pos[slot];
-        }
-        if (pos < 0) continue;
-        if (req < 0 || req >= a.n_req || br < 0 || br >= a.n_branch || pos >= a.n_pos) {
-            if (lane == 0) flag_error(a.err, RPS_DEVERR_ROW_INDEX);
+        issued = __shfl_sync(kFull, issued, 0);
+    };
+
+    int64_t g = g_begin;
+    int64_t r;
+    Segment s;
+    while (next_segment<DT>(a, seg_start, nv, g, g_end, r, s)) {
+        if (!s.valid) {
+            if (s.bad && lane == 0) flag_error(a.err, RPS_DEVERR_ROW_INDEX);
             continue;
         }
-        const char *row = base + (req * a.req_stride + br * a.branch_stride + pos * a.pos_stride) * kBytes;
-
         LaneState L;
-        float tv;
-        int ti;
-        const int V32 = static_cast<int>(a.vocab);
-        scan_segment<DT, TOPK, false>(row, V32, static_cast<int>(u0), static_cast<int>(u1), a.k, lane, L, tv, ti, stage);
+        lane_init(L);
+        typename E::Sketch *sketch = TOPK ? static_cast<typename E::Sketch *>(a.sketch) + s.slot * nv : nullptr;
+        const int cend = min(s.u1, full_units);
+        for (int cu = s.u0; cu < cend; cu += kChunkUnits) {
+            int st;
+            if (!acquire(st)) return;
+            fold_chunk<DT, TOPK>(L, sketch, ring + st * kChunkUnits, min(kChunkUnits, cend - cu), cu, lane);
+            release();
+        }
+        if (s.u1 > full_units) fold_tail<DT, false>(L, s.row, V, lane);
         {
             float a0, a1, b0, b1;
             unpack2(L.s, a0, a1);
             unpack2(L.t, b0, b1);
             const float chk = a0 + a1 + b0 + b1;
             if (__any_sync(kFull, chk != chk)) {
-                scan_segment<DT, TOPK, true>(row, V32, static_cast<int>(u0), static_cast<int>(u1), a.k, lane, L, tv,
-                                             ti, stage);
+                rescan_safe<DT>(L, s.row, V, s.u0, s.u1, lane);
                 if (L.bad) L.s = pack2(NAN, NAN);
             }
         }
         const float MX = warp_max(L.mx);
-        const int am = resolve_argmax<DT>(row, a.vocab, L, MX);
+        const int am = resolve_argmax<DT>(s.row, V, L, MX, lane);
+        float tv = -INFINITY;
+        int ti = INT_MAX;
+        if (TOPK) {
+            // the k-th largest lane maximum bounds the segment's k-th largest logit from below
+            topk_from_sketch<DT>(L, s.row, sketch, s.u0, cend, a.k, lane, warp_kth_largest(L.mx, a.k, lane), tv, ti,
+                                 stage, cand);
+            if (s.u1 > full_units) topk_tail<DT>(s.row, V, a.k, lane, tv, ti);
+        }
         float s_lo, s_hi, t_lo, t_hi;
         unpack2(L.s, s_lo, s_hi);
         unpack2(L.t, t_lo, t_hi);
@@ -547,6 +973,7 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) row_stats_kernel(c
         const int64_t w_first = (r * nv) / piece;
         const int64_t w_last = ((r + 1) * nv - 1) / piece;
         const int count = static_cast<int>(w_last - w_first + 1);
+        const int64_t slot = s.slot;
         if (count == 1) {
             write_row(a, slot, rt, tv, ti, lane);
             continue;
@@ -590,49 +1017,35 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) row_stats_kernel(c
             p.amax = __ldcg(&part[lane].amax);
         }
         rt = combine(p.mref, p.s, p.t, p.mx, p.amax);
-        if (TOPK) {
-            const float2 *lists = a.part_topk + slot * kMaxPartials * a.k;
-            float2 e = __ldcg(lists + lane % a.k);  // list 0 seeds the merged list
-            tv = lane < a.k ? e.x : -INFINITY;
-            ti = lane < a.k ? __float_as_int(e.y) : INT_MAX;
-            const int total_entries = count * a.k;
-            for (int base_e = a.k; base_e < total_entries; base_e += 32) {
-                const int idx = base_e + lane;
-                float cv = -INFINITY;
-                int ci = INT_MAX;
-                if (idx < total_entries) {
-                    const float2 f = __ldcg(lists + idx);
-                    cv = f.x;
-                    ci = __float_as_int(f.y);
-                }
-                float th = __shfl_sync(kFull, tv, a.k - 1);
-                bool has = idx < total_entries && ci != INT_MAX && cv >= th;
-                while (true) {
-                    const unsigned lanes = __ballot_sync(kFull, has);
-                    if (!lanes) break;
-                    const int src = __ffs(lanes) - 1;
-                    const float v = __shfl_sync(kFull, cv, src);
-                    const int i = __shfl_sync(kFull, ci, src);
-                    if (lane == src) has = false;
-                    topk_insert(tv, ti, v, i, a.k, lane);
-                    th = __shfl_sync(kFull, tv, a.k - 1);
-                    has = has && cv >= th;
-                }
-            }
-        }
+        if (TOPK) merge_topk(a.part_topk + slot * kMaxPartials * a.k, count, a.k, lane, tv, ti);
         write_row(a, slot, rt, tv, ti, lane);
     }
 }
 
 template <int DT, bool TOPK>
+constexpr int dyn_smem_bytes() {
+    return kWarps * (kStages * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0)) *
+           static_cast<int>(sizeof(uint4));
+}
+
+template <int DT, bool TOPK>
+cudaError_t prepare_typed() {
+    return cudaFuncSetAttribute(row_stats_kernel<DT, TOPK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                dyn_smem_bytes<DT, TOPK>());
+}
+
+template <int DT, bool TOPK>
 cudaError_t launch_typed(const RowStatsArgs &a, int grid, cudaStream_t stream) {
-    row_stats_kernel<DT, TOPK><<<grid, kRowThreads, 0, stream>>>(a);
+    row_stats_kernel<DT, TOPK><<<grid, kRowThreads, dyn_smem_bytes<DT, TOPK>(), stream>>>(a);
     return cudaGetLastError();
 }
 
 template <int DT, bool TOPK>
 cudaError_t occupancy_typed(int *blocks) {
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK>, kRowThreads, 0);
+    cudaError_t e = prepare_typed<DT, TOPK>();
+    if (e != cudaSuccess) return e;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK>, kRowThreads,
+                                                         dyn_smem_bytes<DT, TOPK>());
 }
 
 }  // namespace

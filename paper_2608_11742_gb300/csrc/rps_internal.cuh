@@ -11,8 +11,15 @@ namespace rps {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kMaxPartials = 32;   // partial records per row (one merging warp)
 constexpr int kRowThreads = 256;   // threads per block of the row-statistics kernel
-constexpr int kRowMinBlocks = 2;  // resident blocks per SM the register budget must allow
-constexpr int kBatch = 4;          // 16-byte vectors a lane loads per batch
+// Shape of each warp's shared-memory ring (overridable at build time for tuning).
+#ifndef RPS_RING_UNITS_PER_LANE
+#define RPS_RING_UNITS_PER_LANE 4
+#endif
+#ifndef RPS_RING_STAGES
+#define RPS_RING_STAGES 2
+#endif
+constexpr int kBatch = RPS_RING_UNITS_PER_LANE;  // 16-byte units a lane takes from each ring buffer
+constexpr int kStages = RPS_RING_STAGES;         // ring buffers (bulk copies in flight) per warp
 
 // Partial statistics of one row segment, base-2 online softmax:
 // s = sum 2^u, t = sum u 2^u with u = (z - mref) * log2(e); mx = max z and
@@ -43,6 +50,7 @@ struct RowStatsArgs {
     // workspace
     Partial *part;        // [slots][kMaxPartials]
     float2 *part_topk;    // [slots][kMaxPartials][k] as (value, index bits)
+    void *sketch;         // [slots][units_per_row] per-(chunk, lane) maxima (top-k mode)
     uint32_t *ticket;     // [slots]
     // decomposition: the rows' 16-byte units are split evenly over `warps` warps
     int64_t units_per_row;
@@ -91,6 +99,7 @@ struct CommitArgs {
 cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream);
 cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream);
 cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream);
+cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStream_t stream);
 
 // ---------------------------------------------------------------- device
 __device__ __forceinline__ void flag_error(uint32_t *err, uint32_t bits) {

@@ -59,7 +59,8 @@ extern "C" rps_status rps_score_step_noalloc(const rps_logits *logits, const rps
     if (rows && rows->n_seg > RPS_MAX_SEGMENTS) return RPS_ERR_UNSUPPORTED;
     if (!arguments_ok(logits, rows, prm, out)) return RPS_ERR_INVALID_ARG;
     const int32_t k = out->topk_idx ? prm->k_max : 0;
-    const size_t need = rps_workspace_bytes(static_cast<int64_t>(rows->n_seg) * rows->cap, logits->vocab, k);
+    const size_t need =
+        rps_workspace_bytes(static_cast<int64_t>(rows->n_seg) * rows->cap, logits->vocab, logits->dtype, k);
     if (need == 0) return RPS_ERR_INVALID_ARG;
     if (need > RPS_STATIC_SCRATCH_BYTES) return RPS_ERR_UNSUPPORTED;  // beyond the fixed scratch
 

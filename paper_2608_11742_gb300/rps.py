@@ -19,7 +19,10 @@ from typing import Optional
 
 import torch
 
-LIB_PATH = Path(__file__).resolve().parent / "librps.so"
+import os
+
+# RPS_LIBRARY selects another build of the library (for example a tuning variant).
+LIB_PATH = Path(os.environ.get("RPS_LIBRARY", Path(__file__).resolve().parent / "librps.so"))
 if not LIB_PATH.exists():
     raise ImportError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
 _lib = C.CDLL(str(LIB_PATH))
@@ -72,7 +75,7 @@ class RpsCommitOut(C.Structure):
 
 
 _lib.rps_workspace_bytes.restype = C.c_size_t
-_lib.rps_workspace_bytes.argtypes = [C.c_int64, C.c_int64, C.c_int32]
+_lib.rps_workspace_bytes.argtypes = [C.c_int64, C.c_int64, C.c_int32, C.c_int32]
 _lib.rps_workspace_init.restype = C.c_int
 _lib.rps_workspace_init.argtypes = [_p, C.c_size_t, _p]
 _lib.rps_score_step.restype = C.c_int
@@ -91,6 +94,10 @@ _lib.rps_score_branches.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.POINTER(R
 _lib.rps_commit.restype = C.c_int
 _lib.rps_commit.argtypes = [C.POINTER(RpsBranchScores), C.c_int32, C.c_int32, C.POINTER(RpsPivots),
                             C.POINTER(RpsParams), C.POINTER(RpsCommitOut), _p]
+_lib.rps_score_and_commit.restype = C.c_int
+_lib.rps_score_and_commit.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.POINTER(RpsRowStats),
+                                      C.POINTER(RpsRowStats), C.c_int32, C.c_int32, C.POINTER(RpsPivots),
+                                      C.POINTER(RpsParams), C.POINTER(RpsBranchScores), C.POINTER(RpsCommitOut), _p]
 _lib.rps_poll_device_status.restype = C.c_int
 _lib.rps_poll_device_status.argtypes = [_p, C.POINTER(C.c_uint32)]
 _lib.rps_status_string.restype = C.c_char_p
@@ -242,8 +249,11 @@ def rps_status_string(status: int) -> str:
     return _lib.rps_status_string(status).decode()
 
 
-def rps_workspace_bytes(max_rows: int, vocab: int, k_max: int) -> int:
-    n = _lib.rps_workspace_bytes(max_rows, vocab, k_max)
+def rps_workspace_bytes(max_rows: int, vocab: int, k_max: int, dtype=RPS_BF16) -> int:
+    """Workspace bytes; dtype is an RPS_* code or a torch dtype of the logits."""
+    if not isinstance(dtype, int):
+        dtype = RPS_BF16 if dtype == torch.bfloat16 else RPS_F32
+    n = _lib.rps_workspace_bytes(max_rows, vocab, dtype, k_max)
     if n == 0:
         raise RPSError(RPS_ERR_INVALID_ARG, "rps_workspace_bytes")
     return n
@@ -298,6 +308,15 @@ def rps_commit(scores: ScoresBuf, n_req: int, L: int, piv: PivotsBuf, prm, out: 
            "rps_commit")
 
 
+def rps_score_and_commit(anchor_logits: torch.Tensor, anchor_branch: int, anchor: RowStatsBuf, branch: RowStatsBuf,
+                         n_req: int, L: int, piv: PivotsBuf, prm, scores: ScoresBuf, out: CommitBuf,
+                         stream=None) -> None:
+    d, a, b, pv, p = logits_desc(anchor_logits), anchor.c(), branch.c(), piv.c(), params(prm)
+    s, o = scores.c(), out.c()
+    _check(_lib.rps_score_and_commit(C.byref(d), anchor_branch, C.byref(a), C.byref(b), n_req, L, C.byref(pv),
+                                     C.byref(p), C.byref(s), C.byref(o), _stream(stream)), "rps_score_and_commit")
+
+
 def rps_poll_device_status(stream=None):
     """Synchronise and return (status, detail bits); clears the device error word."""
     detail = C.c_uint32(0)
@@ -311,12 +330,12 @@ class Step:
 
     The base branch (0) of ``logits`` is the anchor, as in the workloads here.
     Kernels launched per ``run``: row statistics of the masked base rows (top-k
-    mode), pivot selection, row statistics of the lookahead rows, branch
-    scores, commit.
+    mode), pivot selection, row statistics of the lookahead rows, and branch
+    scores with the commit decision in one launch.
     """
-    LAUNCHES = 5
+    LAUNCHES = 4
 
-    def __init__(self, n_req: int, L: int, V: int, prm, device):
+    def __init__(self, n_req: int, L: int, V: int, prm, device, dtype=torch.bfloat16):
         self.n_req, self.L, self.V, self.prm = n_req, L, V, prm
         P, K, k = prm.n_pivots, prm.tokens_per_pivot, prm.k_max
         self.NB = P * K
@@ -325,8 +344,8 @@ class Step:
         self.piv = PivotsBuf.alloc(n_req, L, P, K, device)
         self.scores = ScoresBuf.alloc(n_req, P, K, device)
         self.commit = CommitBuf.alloc(n_req, L, P, device)
-        base_ws = rps_workspace_bytes(n_req * L, V, k)
-        br_ws = rps_workspace_bytes(n_req * self.NB * L, V, 0)
+        base_ws = rps_workspace_bytes(n_req * L, V, k, dtype)
+        br_ws = rps_workspace_bytes(n_req * self.NB * L, V, 0, dtype)
         self.ws_base = torch.empty(base_ws, dtype=torch.uint8, device=device)
         self.ws_branch = torch.empty(br_ws, dtype=torch.uint8, device=device)
         rps_workspace_init(self.ws_base)
@@ -350,9 +369,12 @@ class Step:
     def decide(self, stream=None):
         rps_commit(self.scores, self.n_req, self.L, self.piv, self.prm, self.commit, stream)
 
+    def score_and_decide(self, logits, stream=None):
+        rps_score_and_commit(logits, 0, self.base, self.branch, self.n_req, self.L, self.piv, self.prm, self.scores,
+                             self.commit, stream)
+
     def run(self, logits, mask_pos, mask_cnt, stream=None):
         self.score_base(logits, mask_pos, mask_cnt, stream)
         self.select(mask_pos, mask_cnt, stream)
         self.score_branch_rows(logits, stream)
-        self.score(logits, stream)
-        self.decide(stream)
+        self.score_and_decide(logits, stream)

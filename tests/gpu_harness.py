@@ -186,7 +186,7 @@ class GpuStep:
         self.t = padded_tensor(logits_np, device)
         self.d_mask_pos = torch.from_numpy(mask_pos).to(device)
         self.d_mask_cnt = torch.from_numpy(mask_cnt).to(device)
-        self.step = rps.Step(n_req, L, V, prm, device)
+        self.step = rps.Step(n_req, L, V, prm, device, self.t.dtype)
 
     def run_and_compare(self, what: str = ""):
         prm, o, st = self.prm, self.o, self.step
@@ -197,8 +197,16 @@ class GpuStep:
         st.score_branch_rows(self.t)
         st.score(self.t)
         st.decide()
+        # the fused launch must give exactly the results of the two separate calls
+        fused_sc = rps.ScoresBuf.alloc(self.n_req, P, K, self.t.device)
+        fused_cm = rps.CommitBuf.alloc(self.n_req, self.L, P, self.t.device)
+        rps.rps_score_and_commit(self.t, 0, st.base, st.branch, self.n_req, self.L, st.piv, prm, fused_sc, fused_cm)
         status, detail = rps.rps_poll_device_status()
         assert status == rps.RPS_OK, f"{what}: device error bits {detail:#x}"
+        for name in ("mean_H", "n_tau", "log_a", "score"):
+            assert torch.equal(getattr(fused_sc, name).nan_to_num(-7.0), getattr(st.scores, name).nan_to_num(-7.0)), name
+        for name in ("best_slot", "winner", "commit_pos", "commit_tok", "mask_cnt"):
+            assert torch.equal(getattr(fused_cm, name), getattr(st.commit, name)), name
 
         base_o = o.base_stats(self.logits_np, self.mask_pos, self.mask_cnt, prm.k_max)
         base_g = stats_np(st.base)

@@ -50,14 +50,18 @@ def test_status_strings_and_version(libs):
 def test_workspace_bytes(libs):
     lib = libs["librps.so"]
     lib.rps_workspace_bytes.restype = C.c_size_t
-    lib.rps_workspace_bytes.argtypes = [C.c_int64, C.c_int64, C.c_int32]
-    a = lib.rps_workspace_bytes(256, 126464, 10)
-    b = lib.rps_workspace_bytes(256, 126464, 0)
+    lib.rps_workspace_bytes.argtypes = [C.c_int64, C.c_int64, C.c_int32, C.c_int32]
+    bf16, f32 = 1, 0
+    a = lib.rps_workspace_bytes(256, 126464, bf16, 10)
+    b = lib.rps_workspace_bytes(256, 126464, bf16, 0)
     assert a > b > 0
-    assert lib.rps_workspace_bytes(512, 126464, 10) > a
-    assert lib.rps_workspace_bytes(0, 126464, 10) == 0
-    assert lib.rps_workspace_bytes(16, 0, 10) == 0
-    assert lib.rps_workspace_bytes(16, 100, 33) == 0
+    assert lib.rps_workspace_bytes(256, 126464, f32, 10) > a  # the top-k sketch is element-sized
+    assert lib.rps_workspace_bytes(256, 126464, f32, 0) == b
+    assert lib.rps_workspace_bytes(512, 126464, bf16, 10) > a
+    assert lib.rps_workspace_bytes(0, 126464, bf16, 10) == 0
+    assert lib.rps_workspace_bytes(16, 0, bf16, 10) == 0
+    assert lib.rps_workspace_bytes(16, 100, bf16, 33) == 0
+    assert lib.rps_workspace_bytes(16, 100, 7, 10) == 0
 
 
 def _binding_types():
@@ -74,7 +78,7 @@ def test_host_rejects_bad_arguments(libs):
     rows = r.RpsRowList(fake, None, 1, 32, None, 0)
     prm = r.RpsParams(10, 0.1, 0.9, 0.9, 0.1, 4, 2)
     out = r.RpsRowStats(fake, fake, fake, fake, fake, fake, fake, fake, fake)
-    ws = lib.rps_workspace_bytes(32, 4096, 10)
+    ws = lib.rps_workspace_bytes(32, 4096, r.RPS_BF16, 10)
 
     def score(logits=good_logits, rows=rows, prm=prm, out=out, ws_ptr=fake, ws_bytes=ws):
         return lib.rps_score_step(C.byref(logits), C.byref(rows), C.byref(prm), C.byref(out), ws_ptr, ws_bytes, None)

@@ -110,7 +110,7 @@ def test_row_stats_parity(rps, dtype, V, n, k):
     prm = Params(k_max=k)
     for topk in (True, False):
         buf = rps.RowStatsBuf.alloc(n, k if topk else 0, "cuda")
-        ws = torch.zeros(rps.rps_workspace_bytes(n, V, k if topk else 0), dtype=torch.uint8, device="cuda")
+        ws = torch.zeros(rps.rps_workspace_bytes(n, V, k if topk else 0, t.dtype), dtype=torch.uint8, device="cuda")
         for rep in range(2):  # the second call checks the workspace is left ready
             rps.rps_score_step(t, desc, None, 1, n, prm, buf, ws)
             status, detail = rps.rps_poll_device_status()
@@ -134,7 +134,7 @@ def test_row_stats_mask_form_and_skips(rps):
     t = to_device(synth.bf16_round(z))
     zb = synth.bf16_round(z)
     buf = rps.RowStatsBuf.alloc(n_req * L, k, "cuda")
-    ws = torch.zeros(rps.rps_workspace_bytes(n_req * L, V, k), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(rps.rps_workspace_bytes(n_req * L, V, k, t.dtype), dtype=torch.uint8, device="cuda")
     rps.rps_score_step(t, None, torch.from_numpy(cnt).cuda(), n_req, L, Params(k_max=k), buf, ws,
                        mask_pos=torch.from_numpy(mask_pos).cuda(), mask_branch=1)
     status, detail = rps.rps_poll_device_status()
@@ -152,7 +152,7 @@ def test_row_stats_mask_form_and_skips(rps):
     z2 = rng.standard_normal((3, 2, 4, V)).astype(np.float32)
     t2 = to_device(z2)
     buf2 = rps.RowStatsBuf.alloc(3, 0, "cuda")
-    ws2 = torch.zeros(rps.rps_workspace_bytes(3, V, 0), dtype=torch.uint8, device="cuda")
+    ws2 = torch.zeros(rps.rps_workspace_bytes(3, V, 0, t2.dtype), dtype=torch.uint8, device="cuda")
     rps.rps_score_step(t2, desc, None, 1, 3, Params(k_max=k), buf2, ws2)
     assert rps.rps_poll_device_status()[0] == rps.RPS_OK
     g2 = stats_np(buf2)
@@ -167,7 +167,7 @@ def test_device_errors_are_reported(rps):
     z[0, 0, 2, 7] = np.nan
     t = to_device(z)
     buf = rps.RowStatsBuf.alloc(3, 0, "cuda")
-    ws = torch.zeros(rps.rps_workspace_bytes(3, V, 0), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(rps.rps_workspace_bytes(3, V, 0, t.dtype), dtype=torch.uint8, device="cuda")
     desc = torch.tensor([[0, 0, 0], [0, 0, 9], [0, 0, 2]], dtype=torch.int32, device="cuda")  # pos 9 out of range
     rps.rps_score_step(t, desc, None, 1, 3, Params(), buf, ws)
     status, detail = rps.rps_poll_device_status()
@@ -181,7 +181,7 @@ def test_device_errors_are_reported(rps):
     mpos = torch.arange(4, dtype=torch.int32, device="cuda").view(1, 4)
     buf4 = rps.RowStatsBuf.alloc(4, 0, "cuda")
     z[0, 0, 2, 7] = 0.0
-    ws4 = torch.zeros(rps.rps_workspace_bytes(4, V, 0), dtype=torch.uint8, device="cuda")
+    ws4 = torch.zeros(rps.rps_workspace_bytes(4, V, 0, torch.float32), dtype=torch.uint8, device="cuda")
     rps.rps_score_step(to_device(z), None, cnt, 1, 4, Params(), buf4, ws4, mask_pos=mpos)
     status, detail = rps.rps_poll_device_status()
     assert status == rps.RPS_ERR_DEVICE and detail & rps.DEVERR_MASK
@@ -260,7 +260,7 @@ def test_full_size_sampled(rps, name, w):
     synth.device_fill(logits, w.seed, w.mixture, valid=None if valid is None else torch.from_numpy(valid).cuda())
     mpos, mcnt = w.mask()
     d_mpos, d_mcnt = torch.from_numpy(mpos).cuda(), torch.from_numpy(mcnt).cuda()
-    step = rps.Step(w.n_req, w.L, w.V, prm, "cuda")
+    step = rps.Step(w.n_req, w.L, w.V, prm, "cuda", dt)
     step.run(logits, d_mpos, d_mcnt)
     status, detail = rps.rps_poll_device_status()
     assert status == rps.RPS_OK, hex(detail)

@@ -42,7 +42,7 @@ def test_noalloc_matches_workspace_entry_point(rps, k):
     t = _rows(n, V, 7 + k)
     desc = torch.tensor([[0, 0, i] for i in range(n)], dtype=torch.int32, device="cuda")
     ref = rps.RowStatsBuf.alloc(n, k, "cuda")
-    ws = torch.zeros(rps.rps_workspace_bytes(n, V, k), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(rps.rps_workspace_bytes(n, V, k, t.dtype), dtype=torch.uint8, device="cuda")
     rps.rps_score_step(t, desc, None, 1, n, prm, ref, ws)
     assert rps.rps_poll_device_status()[0] == rps.RPS_OK
     want = stats_np(ref)
@@ -59,7 +59,7 @@ def test_noalloc_rejects_requests_beyond_the_scratch(rps):
     V = 4096
     limit = 8 << 20
     n = 1
-    while rps.rps_workspace_bytes(n, V, 10) <= limit:
+    while rps.rps_workspace_bytes(n, V, 10, torch.bfloat16) <= limit:
         n *= 2
     t = _rows(4, V, 1)
     desc = torch.zeros((n, 3), dtype=torch.int32, device="cuda")
