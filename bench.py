@@ -141,22 +141,26 @@ class Workload:
         self.branch_rows = int(self.step.piv.n_branch_rows.sum())
         self.graph = self._capture()
 
+    KERNELS = ("base_rows_topk", "select", "lookahead_rows", "score_commit")
+
     def _capture(self):
         import torch
         g = torch.cuda.CUDAGraph()
         try:
-            ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+            ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(5)]
         except TypeError:  # torch without external events: time the kernel in its own graph
             ev = None
+        calls = (lambda: self.step.score_base(self.logits, self.mpos, self.mcnt),
+                 lambda: self.step.select(self.mpos, self.mcnt),
+                 lambda: self.step.score_branch_rows(self.logits),
+                 lambda: self.step.score_and_decide(self.logits))
         with torch.cuda.graph(g, stream=self.stream):
-            self.step.score_base(self.logits, self.mpos, self.mcnt)
-            self.step.select(self.mpos, self.mcnt)
+            for i, call in enumerate(calls):
+                if ev:
+                    ev[i].record()
+                call()
             if ev:
-                ev[0].record()
-            self.step.score_branch_rows(self.logits)
-            if ev:
-                ev[1].record()
-            self.step.score_and_decide(self.logits)
+                ev[4].record()
         self.ev = ev
         if ev is None:
             self.k1_graph = torch.cuda.CUDAGraph()
@@ -178,6 +182,7 @@ class Workload:
         s = self.stream
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         step_ms, k1_ms = [], []
+        self.kernel_ms = {k: [] for k in self.KERNELS}
         for i in range(warmup + steps):
             with torch.cuda.stream(s):
                 flush.add_(1)
@@ -188,7 +193,9 @@ class Workload:
             if i >= warmup:
                 step_ms.append(e0.elapsed_time(e1))
                 if self.ev:
-                    k1_ms.append(self.ev[0].elapsed_time(self.ev[1]))
+                    for j, name in enumerate(self.KERNELS):
+                        self.kernel_ms[name].append(self.ev[j].elapsed_time(self.ev[j + 1]))
+                    k1_ms.append(self.kernel_ms["lookahead_rows"][-1])
         if not self.ev:
             for i in range(warmup + steps):
                 with torch.cuda.stream(s):
@@ -329,6 +336,7 @@ def run_gpu(args):
                      "algorithmic_bytes_per_launch": wl.branch_bytes(), "launch_ms": k1},
         "clocks": clocks,
         "gpu_launches": rps.Step.LAUNCHES * args.steps,
+        "kernel_us": {k: statistics.mean(v) * 1e3 for k, v in wl.kernel_ms.items() if v},
     }
     del wl
     torch.cuda.empty_cache()
@@ -342,6 +350,7 @@ def run_gpu(args):
             ts = statistics.mean(sm)
             kk = statistics.mean(km)
             others[name] = {"rows_per_step": x.rows(), "step_us": ts * 1e3, "p50_step_us": statistics.median(sm) * 1e3,
+                            "kernel_us": {k: statistics.mean(v) * 1e3 for k, v in x.kernel_ms.items() if v},
                             "p90_step_us": sorted(sm)[int(0.9 * (len(sm) - 1))] * 1e3,
                             "rows_per_s": x.rows() / (ts / 1e3), "gbs": x.bytes() / (ts / 1e3) / 1e9,
                             "frac": x.bytes() / (ts / 1e3) / 1e9 / peak,

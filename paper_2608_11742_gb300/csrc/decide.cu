@@ -81,6 +81,8 @@ __device__ Best block_best(Best mine, Best *buf) {
 constexpr int kSelectBytesPerPos = 3 * sizeof(float) + 3 * sizeof(int32_t) + 2;
 
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs a) {
+    pdl_wait();
+    pdl_launch_next();
     const int q = blockIdx.x;
     const int tid = threadIdx.x;
     const int L = a.L, P = a.P, K = a.K, NB = P * K;
@@ -433,6 +435,8 @@ __device__ void commit_request(const CommitArgs &a, int q, const float *s_req) {
 }
 
 __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a) {
+    pdl_wait();
+    pdl_launch_next();
     __shared__ PivotView v;
     stage_pivots(a.piv, blockIdx.x, a.P, v);
     __syncthreads();
@@ -440,11 +444,15 @@ __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a)
 }
 
 __global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
+    pdl_wait();
+    pdl_launch_next();
     const int q = blockIdx.x;
     commit_request(a, q, a.score + static_cast<int64_t>(q) * a.P * (a.K + 1));
 }
 
 __global__ void __launch_bounds__(kScoreThreads) score_commit_kernel(const ScoreArgs s, const CommitArgs c) {
+    pdl_wait();
+    pdl_launch_next();
     __shared__ PivotView v;
     __shared__ float sc[kMaxSlots];
     stage_pivots(s.piv, blockIdx.x, s.P, v);
@@ -463,23 +471,19 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream) {
             cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
         if (e != cudaSuccess) return e;
     }
-    select_kernel<<<a.n_req, kSelectThreads, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(select_kernel, dim3(a.n_req), dim3(kSelectThreads), smem, stream, a);
 }
 
 cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream) {
-    score_kernel<<<a.n_req, kScoreThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(score_kernel, dim3(a.n_req), dim3(kScoreThreads), 0, stream, a);
 }
 
 cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream) {
-    commit_kernel<<<a.n_req, 32, 0, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(commit_kernel, dim3(a.n_req), dim3(32), 0, stream, a);
 }
 
 cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStream_t stream) {
-    score_commit_kernel<<<s.n_req, kScoreThreads, 0, stream>>>(s, c);
-    return cudaGetLastError();
+    return launch_pdl(score_commit_kernel, dim3(s.n_req), dim3(kScoreThreads), 0, stream, s, c);
 }
 
 }  // namespace rps

@@ -816,6 +816,8 @@ __global__ void __launch_bounds__(kRowThreads, 4) row_stats_kernel(const RowStat
     constexpr int kRing = kStages;
     __shared__ __align__(8) uint64_t bars[kWarps][kRing];
 
+    pdl_wait();
+    pdl_launch_next();
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
     const int warp = blockIdx.x * kWarps + wib;
@@ -1036,8 +1038,7 @@ cudaError_t prepare_typed() {
 
 template <int DT, bool TOPK>
 cudaError_t launch_typed(const RowStatsArgs &a, int grid, cudaStream_t stream) {
-    row_stats_kernel<DT, TOPK><<<grid, kRowThreads, dyn_smem_bytes<DT, TOPK>(), stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(row_stats_kernel<DT, TOPK>, dim3(grid), dim3(kRowThreads), dyn_smem_bytes<DT, TOPK>(), stream, a);
 }
 
 template <int DT, bool TOPK>

@@ -2,6 +2,8 @@
 #pragma once
 
 #include <cstdint>
+#include <utility>
+
 #include <cuda_runtime.h>
 
 #include "rps.h"
@@ -100,6 +102,34 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream);
 cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream);
 cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream);
 cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStream_t stream);
+
+// ---------------------------------------------------------------- launches
+// Every kernel of the library is launched with programmatic stream
+// serialization: it may start while the previous kernel on the stream finishes,
+// and waits (pdl_wait) for that kernel's completion and memory before reading
+// anything. When the previous kernel is not one of ours this is the ordinary
+// stream order.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// Waits until the previous kernel on the stream has completed and its writes are visible.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Lets the next kernel on the stream begin launching (it still waits in pdl_wait).
+__device__ __forceinline__ void pdl_launch_next() { asm volatile("griddepcontrol.launch_dependents;" :::); }
 
 // ---------------------------------------------------------------- device
 __device__ __forceinline__ void flag_error(uint32_t *err, uint32_t bits) {
