@@ -8,11 +8,15 @@ selection, row statistics of the lookahead rows, benefit scores and the commit
 decision. The headline workload is one generation step: 256 masked positions,
 vocab 126,464, bf16 logits, 1 base + 8 lookahead branches (4 pivots x top-2).
 
-Timing: the five launches of a step are captured in one CUDA graph; each timed
-replay is preceded by a 256 MB write that flushes L2 and bracketed by CUDA
-events on the launching stream; event nodes inside the graph time the lookahead
-row-statistics kernel (the dominant kernel) on the same stream. SM clocks and
-throttle reasons are sampled with nvidia-smi during the timed region.
+Timing: the launches of a step are captured in one CUDA graph; each timed
+replay is preceded by an L2 flush (a 256 MB buffer is written, then read back,
+so that L2 holds none of the step's data and no dirty lines whose write-back
+would land inside the timed region) and bracketed by CUDA events on the
+launching stream; event nodes inside the graph time each kernel, including the
+lookahead row-statistics kernel (the dominant kernel), on the same stream. SM
+clocks and throttle reasons are sampled with nvidia-smi during the timed region.
+The roofline's `traffic` (DRAM bytes of one launch, from ncu) is reported only
+while the kernel sources hash to the value recorded beside it.
 
 `value` is scored logit rows per second over the whole job (N replicas, one per
 GPU, no collective in the data path: weak scaling). `e2e` is the same metric
@@ -41,6 +45,42 @@ HEADLINE = "step"
 OTHERS = ("step-50", "step-10", "long", "block", "serve")
 FLUSH_BYTES = 256 << 20
 FALLBACK_HBM_GBS = 6800.0
+KERNEL_SOURCES = ("paper_2608_11742_gb300/csrc/rowstats.cu", "paper_2608_11742_gb300/csrc/rps_internal.cuh")
+
+
+class L2Flush:
+    """Write a buffer larger than L2, then read it back: the read evicts the
+    written lines (their write-back happens here, outside the timed region) and
+    leaves only clean lines of the flush buffer in L2."""
+
+    def __init__(self, device):
+        import torch
+        self.buf = torch.zeros(FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+        self.sink = torch.zeros((), dtype=torch.float32, device=device)
+
+    def __call__(self):
+        import torch
+        self.buf.add_(1)
+        torch.sum(self.buf, dim=0, out=self.sink)
+
+
+def kernel_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        h.update((ROOT / rel).read_bytes())
+    return h.hexdigest()
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the lookahead kernel, if recorded for the current sources."""
+    tf = ROOT / "profiles" / "traffic.json"
+    if not tf.exists():
+        return None
+    d = json.loads(tf.read_text())
+    if d.get("source_sha256") != kernel_source_hash():
+        return None
+    return d.get("workloads", {}).get(workload)
 
 
 def describe(w) -> str:
@@ -185,7 +225,7 @@ class Workload:
         self.kernel_ms = {k: [] for k in self.KERNELS}
         for i in range(warmup + steps):
             with torch.cuda.stream(s):
-                flush.add_(1)
+                flush()
                 e0.record(s)
                 self.graph.replay()
                 e1.record(s)
@@ -199,7 +239,7 @@ class Workload:
         if not self.ev:
             for i in range(warmup + steps):
                 with torch.cuda.stream(s):
-                    flush.add_(1)
+                    flush()
                     e0.record(s)
                     self.k1_graph.replay()
                     e1.record(s)
@@ -291,7 +331,7 @@ def run_gpu(args):
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    flush = torch.zeros(FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    flush = L2Flush(device)
     peak, peak_kind = peaks()
 
     w = configs.ALL[args.workload]
@@ -312,11 +352,7 @@ def run_gpu(args):
     value = world * rows / (t_step / 1e3)
     k1 = statistics.mean(k1_ms)
     achieved = wl.branch_bytes() / (k1 / 1e3) / 1e9
-    traffic = None
-    tf = ROOT / "profiles" / "traffic.json"
-    if tf.exists():
-        d = json.loads(tf.read_text())
-        traffic = d.get(args.workload)
+    traffic = recorded_traffic(args.workload)
 
     out = {
         "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
@@ -326,7 +362,7 @@ def run_gpu(args):
                    "params": {"k_max": prm.k_max, "r": prm.r, "tau_pivot": prm.tau_pivot, "tau": prm.tau,
                               "lambda": prm.lam, "n_pivots": prm.n_pivots, "tokens_per_pivot": prm.tokens_per_pivot},
                    "rows_per_step": rows, "base_rows": wl.base_rows, "lookahead_rows": wl.branch_rows,
-                   "bytes_per_step": wl.bytes(), "l2": "flushed (256 MB write) before every timed step",
+                   "bytes_per_step": wl.bytes(), "l2": "flushed before every timed step (256 MB buffer written, then read back)",
                    "parallelism": f"{world} independent replica(s), no collective"},
         "achieved_gbs": wl.bytes() / (t_step / 1e3) / 1e9,
         "frac_of_hbm_peak": wl.bytes() / (t_step / 1e3) / 1e9 / peak,
