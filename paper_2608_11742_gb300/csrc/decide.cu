@@ -52,10 +52,12 @@ struct Best {
     int idx;
 };
 
+// Larger value first, then lower position; the entry index makes the order
+// total (positions are distinct in valid input).
 __device__ __forceinline__ bool better(const Best &a, const Best &b) {
     if (a.idx < 0) return false;
     if (b.idx < 0) return true;
-    return a.v > b.v || (a.v == b.v && a.pos < b.pos);
+    return a.v > b.v || (a.v == b.v && (a.pos < b.pos || (a.pos == b.pos && a.idx < b.idx)));
 }
 
 __device__ Best block_best(Best mine, Best *buf) {
@@ -77,8 +79,26 @@ __device__ Best block_best(Best mine, Best *buf) {
     return r;
 }
 
+// Pivot order as one unsigned key: larger truncated entropy first, then lower
+// position (positions are distinct). The float's bits are mapped to an unsigned
+// order; 0 is below every key and marks "none".
+__device__ __forceinline__ uint64_t pivot_key(float v, int pos) {
+    const uint32_t b = __float_as_uint(v + 0.f);  // -0 orders as +0
+    const uint32_t hi = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return (static_cast<uint64_t>(hi) << 32) | static_cast<uint32_t>(~pos);
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const uint64_t w = __shfl_xor_sync(kFull, v, o);
+        v = w > v ? w : v;
+    }
+    return v;
+}
+
 // Dynamic shared memory of select_kernel per masked position.
-constexpr int kSelectBytesPerPos = 3 * sizeof(float) + 3 * sizeof(int32_t) + 2;
+constexpr int kSelectBytesPerPos = 3 * sizeof(uint64_t) + 3 * sizeof(float) + 4 * sizeof(int32_t) + 2;
 
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs a) {
     pdl_wait();
@@ -93,29 +113,38 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
     __shared__ Best best_buf[kSelectThreads / 32];
     __shared__ int piv_i[RPS_MAX_PIVOTS];  // index of pivot j in M'
     __shared__ int piv_nc[RPS_MAX_PIVOTS];
+    __shared__ uint64_t winners[RPS_MAX_PIVOTS];
+    __shared__ int n_piv_s;
+    __shared__ int br_off[RPS_MAX_PIVOTS * RPS_MAX_K + 1];
+    __shared__ int16_t valid_b[RPS_MAX_PIVOTS * RPS_MAX_K];  // the m-th valid branch
     extern __shared__ __align__(16) unsigned char sel_smem[];
-    float *pm = reinterpret_cast<float *>(sel_smem);  // P^max of mask entry k
+    uint64_t *keys = reinterpret_cast<uint64_t *>(sel_smem);  // pivot key of M' entry i (0: infeasible)
+    uint64_t *t_a = keys + L;                           // tournament buffers
+    uint64_t *t_b = t_a + L;
+    float *pm = reinterpret_cast<float *>(t_b + L);    // P^max of mask entry k
     float *mu = pm + L;                                // retained mass
     float *ht = mu + L;                                // truncated entropy
     int32_t *pos = reinterpret_cast<int32_t *>(ht + L);  // position
     int32_t *am = pos + L;                               // argmax token
     int32_t *rk = am + L;                                // M' entry i -> mask entry
-    uint8_t *in_S = reinterpret_cast<uint8_t *>(rk + L);
+    int32_t *rp = rk + L;                                // M' entry i -> position
+    uint8_t *in_S = reinterpret_cast<uint8_t *>(rp + L);
     uint8_t *taken = in_S + L;
 
+    // Stage this request's statistics over the whole capacity, so that these
+    // loads do not wait for the mask count (entries past it are never used),
+    // and write the defaults.
     int cnt = a.mask_cnt[q];
-    if (cnt < 0 || cnt > L) {
-        if (tid == 0) flag_error(a.err, RPS_DEVERR_MASK);
-        cnt = cnt < 0 ? 0 : L;
-    }
-
-    // Stage this request's statistics (independent loads) and write the defaults.
-    for (int k = tid; k < cnt; k += blockDim.x) {
+    for (int k = tid; k < L; k += blockDim.x) {
         pm[k] = a.pmax[base + k];
         mu[k] = a.mu[base + k];
         ht[k] = a.htrunc[base + k];
         pos[k] = a.mask_pos[base + k];
         am[k] = a.argmax[base + k];
+    }
+    if (cnt < 0 || cnt > L) {
+        if (tid == 0) flag_error(a.err, RPS_DEVERR_MASK);
+        cnt = cnt < 0 ? 0 : L;
     }
     for (int j = tid; j < P; j += blockDim.x) {
         o.pivot_k[q * P + j] = -1;
@@ -164,6 +193,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
             } else {
                 const int r = k - (n_commit + excl);
                 rk[r] = k;
+                rp[r] = pos[k];
+                keys[r] = mu[k] >= a.tau_pivot && ht[k] == ht[k] ? pivot_key(ht[k], pos[k]) : 0ull;
                 o.rem_k[base + r] = k;
                 o.rem_pos[base + r] = pos[k];
             }
@@ -183,46 +214,83 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
     for (int i = tid; i < n_rem; i += blockDim.x) taken[i] = 0;
     __syncthreads();
 
-    // Steps 3-4: feasibility (mu >= tau_pivot) and pivots by truncated entropy.
-    int n_piv = 0;
-    for (int j = 0; j < P; ++j) {
-        Best mine{-INFINITY, INT_MAX, -1};
-        for (int i = tid; i < n_rem; i += blockDim.x) {
-            const int k = rk[i];
-            if (taken[i] || !(mu[k] >= a.tau_pivot)) continue;
-            Best c{ht[k], pos[k], i};
-            if (!(c.v == c.v)) continue;
-            if (better(c, mine)) mine = c;
+    // Steps 3-4: feasibility (mu >= tau_pivot) and the P best feasible rows by
+    // truncated entropy (descending, lower position on ties), as a tournament on
+    // the keys: in every group of 32, each key counts the larger keys of its group
+    // and the P best move on, until one group is left. Keys are distinct (0, the
+    // infeasible mark, excepted), so ranks are too.
+    {
+        const uint64_t *cur = keys;
+        uint64_t *nxt = t_a;
+        int count = n_rem;
+        for (;;) {
+            const int groups = (count + 31) / 32;
+            uint64_t *dst = groups == 1 ? winners : nxt;
+            const int n_dst = groups == 1 ? P : groups * P;
+            for (int t = tid; t < n_dst; t += blockDim.x) dst[t] = 0ull;
+            __syncthreads();
+            for (int t = tid; t < count; t += blockDim.x) {
+                const uint64_t me = cur[t];
+                if (me == 0ull) continue;
+                const int g0 = t & ~31, g1 = min(count, g0 + 32);
+                int rank = 0;
+                for (int u = g0; u < g1; ++u) rank += cur[u] > me;
+                if (rank < P) dst[(t >> 5) * P + rank] = me;
+            }
+            __syncthreads();
+            if (groups == 1) break;
+            cur = nxt;
+            nxt = nxt == t_a ? t_b : t_a;
+            count = groups * P;
         }
-        const Best b = block_best(mine, best_buf);
-        if (b.idx < 0) break;
         if (tid == 0) {
-            taken[b.idx] = 1;
-            piv_i[j] = b.idx;
-            o.pivot_k[q * P + j] = rk[b.idx];
-            o.pivot_pos[q * P + j] = b.pos;
+            int c = 0;
+            while (c < P && winners[c] != 0ull) ++c;
+            n_piv_s = c;
         }
-        n_piv = j + 1;
+        __syncthreads();
+        for (int i = tid; i < n_rem; i += blockDim.x) {
+            const uint64_t key = keys[i];
+            if (key == 0ull) continue;
+            for (int j = 0; j < n_piv_s; ++j) {
+                if (key == winners[j]) {
+                    piv_i[j] = i;
+                    o.pivot_k[q * P + j] = rk[i];
+                    o.pivot_pos[q * P + j] = rp[i];
+                }
+            }
+        }
         __syncthreads();
     }
+    const int n_piv = n_piv_s;
     if (n_piv == 0) {
         if (tid == 0) o.state[q] = RPS_STATE_NO_FEASIBLE;
         return;
     }
 
-    // Step 5: candidates z_v - zmax >= log r in rank order, at most K.
-    if (tid < n_piv) {
-        const int j = tid;
-        const int64_t row = base + rk[piv_i[j]];
-        const double zmax = a.zmax[row];
-        int nc = 0;
-        for (int t = 0; t < a.k_max && nc < K; ++t) {
-            const double zt = a.topk_logit[row * a.k_max + t];
-            if (zt - zmax >= a.log_r)
-                o.cand_tok[(static_cast<int64_t>(q) * P + j) * K + nc++] = a.topk_idx[row * a.k_max + t];
+    // Step 5: candidates z_v - zmax >= log r in rank order, at most K: one warp
+    // per pivot, lane t tests rank t of T_i (all loads at once).
+    {
+        const int lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
+        for (int j = w; j < n_piv; j += nw) {
+            const int64_t row = base + rk[piv_i[j]];
+            const double zmax = a.zmax[row];
+            bool pass = false;
+            int tok = -1;
+            if (lane < a.k_max) {
+                const double zt = a.topk_logit[row * a.k_max + lane];
+                tok = a.topk_idx[row * a.k_max + lane];
+                pass = zt - zmax >= a.log_r;
+            }
+            const unsigned m = __ballot_sync(kFull, pass);
+            const int rank = __popc(m & ((1u << lane) - 1u));
+            if (pass && rank < K) o.cand_tok[(static_cast<int64_t>(q) * P + j) * K + rank] = tok;
+            if (lane == 0) {
+                const int nc = min(__popc(m), K);
+                piv_nc[j] = nc;
+                o.n_cand[q * P + j] = nc;
+            }
         }
-        piv_nc[j] = nc;
-        o.n_cand[q * P + j] = nc;
     }
     __syncthreads();
     int searchable = 0;
@@ -232,36 +300,42 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         return;
     }
 
-    // Step 6: branch b = j * K + c lists M' without pivot j.
-    int off = 0;
-    for (int j = 0; j < P; ++j) {
-        const bool searched = j < n_piv && piv_nc[j] >= 2;
-        for (int c = 0; c < K; ++c) {
-            const int b = j * K + c;
-            const bool valid = searched && c < piv_nc[j];
+    // Step 6: branch b = j * K + c lists M' without pivot j; the lists of the
+    // valid branches are laid end to end in branch order.
+    if (tid == 0) {
+        int off = 0, m = 0;
+        for (int b = 0; b < NB; ++b) {
+            const int j = b / K, c = b % K;
+            const bool valid = j < n_piv && piv_nc[j] >= 2 && c < piv_nc[j];
             const int n = valid ? n_rem - 1 : 0;
-            if (tid == 0) {
-                o.branch_off[q * NB + b] = off;
-                o.branch_cnt[q * NB + b] = n;
-                o.branch_valid[q * NB + b] = valid;
-            }
-            if (valid) {
-                const int pi = piv_i[j];
-                int32_t *rows = o.branch_rows + (static_cast<int64_t>(q) * NB * L + off) * 3;
-                for (int i = tid; i < n_rem; i += blockDim.x) {
-                    if (i == pi) continue;
-                    const int d = i < pi ? i : i - 1;
-                    rows[d * 3 + 0] = q;
-                    rows[d * 3 + 1] = 1 + b;
-                    rows[d * 3 + 2] = pos[rk[i]];
-                }
-            }
+            if (valid) valid_b[m++] = static_cast<int16_t>(b);
+            br_off[b] = off;
+            o.branch_off[q * NB + b] = off;
+            o.branch_cnt[q * NB + b] = n;
+            o.branch_valid[q * NB + b] = valid;
             off += n;
         }
-    }
-    if (tid == 0) {
+        br_off[NB] = off;
         o.n_branch_rows[q] = off;
         o.state[q] = RPS_STATE_SEARCH;
+    }
+    __syncthreads();
+    // one warp per valid branch: M' in order, without the branch's pivot
+    {
+        const int lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
+        const int n_valid = n_rem > 1 ? br_off[NB] / (n_rem - 1) : 0;
+        for (int m = w; m < n_valid; m += nw) {
+            const int b = valid_b[m];
+            const int pi = piv_i[b / K];
+            int32_t *rows = o.branch_rows + (static_cast<int64_t>(q) * NB * L + br_off[b]) * 3;
+            // the (q, 1 + b, pos) triples as consecutive words: contiguous stores
+            const int n_words = (n_rem - 1) * 3;
+            for (int x = lane; x < n_words; x += 32) {
+                const int d = x / 3, f = x - d * 3;
+                const int i = d < pi ? d : d + 1;
+                rows[x] = f == 0 ? q : f == 1 ? 1 + b : rp[i];
+            }
+        }
     }
 }
 
@@ -271,15 +345,27 @@ __device__ __forceinline__ float load_logit(const void *data, int dtype, int64_t
     return static_cast<const float *>(data)[e];
 }
 
-// Pivot-selection facts of one request, staged in shared memory.
+// Pivot-selection facts of one request, staged in shared memory with
+// independent loads so that the scoring and the decision need no further
+// dependent global round trips.
 struct PivotView {
     int state, n_rem;
     int pivot_k[RPS_MAX_PIVOTS];
     int pivot_pos[RPS_MAX_PIVOTS];
     int n_cand[RPS_MAX_PIVOTS];
+    int branch_off[RPS_MAX_PIVOTS * RPS_MAX_K];
+    int branch_cnt[RPS_MAX_PIVOTS * RPS_MAX_K];
+    int cand_tok[RPS_MAX_PIVOTS * RPS_MAX_K];
+    uint8_t branch_valid[RPS_MAX_PIVOTS * RPS_MAX_K];
 };
 
-__device__ void stage_pivots(const rps_pivots &pv, int q, int P, PivotView &v) {
+// Dynamic shared memory of the score / commit kernels: rem_k and rem_pos of one request.
+__host__ __device__ constexpr size_t view_smem_bytes(int L) { return 2 * static_cast<size_t>(L) * sizeof(int32_t); }
+
+__device__ void stage_view(const rps_pivots &pv, int q, int L, int P, int K, PivotView &v, int32_t *rem_k,
+                           int32_t *rem_pos) {
+    const int NB = P * K;
+    const int64_t base = static_cast<int64_t>(q) * L;
     if (threadIdx.x == 0) {
         v.state = pv.state[q];
         v.n_rem = pv.rem_cnt[q];
@@ -289,50 +375,62 @@ __device__ void stage_pivots(const rps_pivots &pv, int q, int P, PivotView &v) {
         v.pivot_pos[j] = pv.pivot_pos[q * P + j];
         v.n_cand[j] = pv.n_cand[q * P + j];
     }
+    for (int b = threadIdx.x; b < NB; b += blockDim.x) {
+        v.branch_valid[b] = pv.branch_valid[q * NB + b];
+        v.branch_off[b] = pv.branch_off[q * NB + b];
+        v.branch_cnt[b] = pv.branch_cnt[q * NB + b];
+        v.cand_tok[b] = pv.cand_tok[static_cast<int64_t>(q) * NB + b];
+    }
+    // the whole capacity: entries past rem_cnt are read but never used
+    for (int i = threadIdx.x; i < L; i += blockDim.x) {
+        rem_k[i] = pv.rem_k[base + i];
+        rem_pos[i] = pv.rem_pos[base + i];
+    }
 }
 
 // Eq. 4 scores of one request, one warp per (pivot, slot); also kept in `sc`.
-__device__ void score_request(const ScoreArgs &a, int q, const PivotView &v, float *sc) {
+__device__ void score_request(const ScoreArgs &a, int q, const PivotView &v, const int32_t *rem_k, float *sc) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
     const int L = a.L, P = a.P, K = a.K, NB = P * K;
     const int64_t base = static_cast<int64_t>(q) * L;
-    const rps_pivots &pv = a.piv;
+    int n_rem = v.n_rem;
+    if (n_rem < 0 || n_rem > L) n_rem = 0;  // select flags bad counts; never index past the capacity
     for (int slot = w; slot < P * (K + 1); slot += nw) {
         const int j = slot / (K + 1), c = slot % (K + 1);
         const int64_t o = (static_cast<int64_t>(q) * P + j) * (K + 1) + c;
         const int pk = v.pivot_k[j];
         float mean_H = NAN, log_a = NAN, score = NAN;
         int n_tau = -1;
-        bool scored = v.state == RPS_STATE_SEARCH && pk >= 0 && v.n_cand[j] >= 2;
-        if (scored && c < K) scored = pv.branch_valid[q * NB + j * K + c] != 0;
+        bool scored = v.state == RPS_STATE_SEARCH && pk >= 0 && pk < L && v.n_cand[j] >= 2;
+        if (scored && c < K) scored = v.branch_valid[j * K + c] != 0;
         if (scored) {
             float sum = 0.f;
             int count = 0;
             float la;
             if (c < K) {
                 const int b = j * K + c;
-                const int64_t first = static_cast<int64_t>(q) * NB * L + pv.branch_off[q * NB + b];
-                const int n = pv.branch_cnt[q * NB + b];
+                const int64_t first = static_cast<int64_t>(q) * NB * L + v.branch_off[b];
+                const int n = v.branch_cnt[b];
+                const int tok = v.cand_tok[b];
+                const int p = v.pivot_pos[j];
+                float z = NAN;
+                if (tok < 0 || tok >= a.vocab) {
+                    if (lane == 0) flag_error(a.err, RPS_DEVERR_TOKEN);
+                } else if (p < 0 || p >= a.n_pos) {
+                    if (lane == 0) flag_error(a.err, RPS_DEVERR_ROW_INDEX);
+                } else {
+                    z = load_logit(a.anchor_data, a.dtype, q * a.req_stride + a.branch_offset + p * a.pos_stride + tok);
+                }
+                const float lse = a.a_lse[base + pk];
                 for (int i = lane; i < n; i += 32) {
                     sum += a.b_H[first + i];
                     count += a.b_pmax[first + i] >= a.tau;
                 }
-                const int tok = pv.cand_tok[(static_cast<int64_t>(q) * P + j) * K + c];
-                const int p = v.pivot_pos[j];
-                if (tok < 0 || tok >= a.vocab) {
-                    if (lane == 0) flag_error(a.err, RPS_DEVERR_TOKEN);
-                    la = NAN;
-                } else if (p < 0 || p >= a.n_pos) {
-                    if (lane == 0) flag_error(a.err, RPS_DEVERR_ROW_INDEX);
-                    la = NAN;
-                } else {
-                    const int64_t e = q * a.req_stride + a.branch_offset + p * a.pos_stride + tok;
-                    la = load_logit(a.anchor_data, a.dtype, e) - a.a_lse[base + pk];
-                }
+                la = z - lse;
             } else {
-                for (int i = lane; i < v.n_rem; i += 32) {
-                    const int k = pv.rem_k[base + i];
-                    if (k == pk) continue;
+                for (int i = lane; i < n_rem; i += 32) {
+                    const int k = rem_k[i];
+                    if (k == pk || k < 0 || k >= L) continue;
                     sum += a.a_H[base + k];
                     count += a.a_pmax[base + k] >= a.tau;
                 }
@@ -340,7 +438,7 @@ __device__ void score_request(const ScoreArgs &a, int q, const PivotView &v, flo
             }
             sum = warp_sum(sum);
             count = warp_sum_int(count);
-            const int n = v.n_rem - 1;
+            const int n = n_rem - 1;
             mean_H = n > 0 ? sum / static_cast<float>(n) : 0.f;
             n_tau = count;
             log_a = la;
@@ -356,28 +454,28 @@ __device__ void score_request(const ScoreArgs &a, int q, const PivotView &v, flo
     }
 }
 
-// Commit decision of one request by one warp; `s` holds the request's scores.
-__device__ void commit_request(const CommitArgs &a, int q, const float *s_req) {
+// Commit decision of one request by one warp; `s_req` holds the request's scores.
+__device__ void commit_request(const CommitArgs &a, int q, const PivotView &v, const int32_t *rem_pos,
+                               const float *s_req) {
     const int lane = threadIdx.x & 31;
-    const int L = a.L, P = a.P, K = a.K, NB = P * K;
+    const int L = a.L, P = a.P, K = a.K;
     const int64_t base = static_cast<int64_t>(q) * L;
-    const rps_pivots &pv = a.piv;
-    const int state = pv.state[q];
+    const int state = v.state;
 
     // Best slot and gain of the pivot held by this lane.
     int best = -1;
     float gain = NAN;
     int ppos = INT_MAX;
     bool wins = false;
-    if (lane < P && state == RPS_STATE_SEARCH && pv.pivot_pos[q * P + lane] >= 0 && pv.n_cand[q * P + lane] >= 2) {
+    if (lane < P && state == RPS_STATE_SEARCH && v.pivot_pos[lane] >= 0 && v.n_cand[lane] >= 2) {
         const float *s = s_req + lane * (K + 1);
         best = K;
         for (int c = 0; c < K; ++c) {
-            if (!pv.branch_valid[q * NB + lane * K + c]) continue;
+            if (!v.branch_valid[lane * K + c]) continue;
             if (s[c] > s[best]) best = c;
         }
         gain = s[best] - s[K];
-        ppos = pv.pivot_pos[q * P + lane];
+        ppos = v.pivot_pos[lane];
         wins = best < K && gain > 0.f;
     }
     if (lane < P) {
@@ -409,8 +507,8 @@ __device__ void commit_request(const CommitArgs &a, int q, const float *s_req) {
         else if (j < 0) winner = RPS_WIN_ANCHOR;
         else {
             winner = j * K + win_best;
-            commit_pos = pv.pivot_pos[q * P + j];
-            ctok = pv.cand_tok[(static_cast<int64_t>(q) * P + j) * K + win_best];
+            commit_pos = v.pivot_pos[j];
+            ctok = v.cand_tok[j * K + win_best];
             margin = g;
         }
         a.out.winner[q] = winner;
@@ -421,11 +519,12 @@ __device__ void commit_request(const CommitArgs &a, int q, const float *s_req) {
     commit_pos = __shfl_sync(kFull, commit_pos, 0);
 
     // Mask after the step: M' without the committed pivot, in order.
-    const int n_rem = state == RPS_STATE_DONE ? 0 : pv.rem_cnt[q];
+    int n_rem = state == RPS_STATE_DONE ? 0 : v.n_rem;
+    if (n_rem < 0 || n_rem > L) n_rem = 0;
     int kept = 0;
     for (int i0 = 0; i0 < n_rem; i0 += 32) {
         const int i = i0 + lane;
-        const int32_t rp = i < n_rem ? pv.rem_pos[base + i] : -1;
+        const int32_t rp = i < n_rem ? rem_pos[i] : -1;
         const bool keep = i < n_rem && rp != commit_pos;
         const unsigned m = __ballot_sync(kFull, keep);
         if (keep) a.out.mask_pos[base + kept + __popc(m & ((1u << lane) - 1u))] = rp;
@@ -438,16 +537,24 @@ __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a)
     pdl_wait();
     pdl_launch_next();
     __shared__ PivotView v;
-    stage_pivots(a.piv, blockIdx.x, a.P, v);
+    extern __shared__ __align__(16) int32_t view_smem[];
+    stage_view(a.piv, blockIdx.x, a.L, a.P, a.K, v, view_smem, view_smem + a.L);
     __syncthreads();
-    score_request(a, blockIdx.x, v, nullptr);
+    score_request(a, blockIdx.x, v, view_smem, nullptr);
 }
 
-__global__ void __launch_bounds__(32) commit_kernel(const CommitArgs a) {
+__global__ void __launch_bounds__(kScoreThreads) commit_kernel(const CommitArgs a) {
     pdl_wait();
     pdl_launch_next();
+    __shared__ PivotView v;
+    __shared__ float sc[kMaxSlots];
+    extern __shared__ __align__(16) int32_t view_smem[];
     const int q = blockIdx.x;
-    commit_request(a, q, a.score + static_cast<int64_t>(q) * a.P * (a.K + 1));
+    stage_view(a.piv, q, a.L, a.P, a.K, v, view_smem, view_smem + a.L);
+    for (int i = threadIdx.x; i < a.P * (a.K + 1); i += blockDim.x)
+        sc[i] = a.score[static_cast<int64_t>(q) * a.P * (a.K + 1) + i];
+    __syncthreads();
+    if (threadIdx.x < 32) commit_request(a, q, v, view_smem + a.L, sc);
 }
 
 __global__ void __launch_bounds__(kScoreThreads) score_commit_kernel(const ScoreArgs s, const CommitArgs c) {
@@ -455,11 +562,12 @@ __global__ void __launch_bounds__(kScoreThreads) score_commit_kernel(const Score
     pdl_launch_next();
     __shared__ PivotView v;
     __shared__ float sc[kMaxSlots];
-    stage_pivots(s.piv, blockIdx.x, s.P, v);
+    extern __shared__ __align__(16) int32_t view_smem[];
+    stage_view(s.piv, blockIdx.x, s.L, s.P, s.K, v, view_smem, view_smem + s.L);
     __syncthreads();
-    score_request(s, blockIdx.x, v, sc);
+    score_request(s, blockIdx.x, v, view_smem, sc);
     __syncthreads();
-    if (threadIdx.x < 32) commit_request(c, blockIdx.x, sc);
+    if (threadIdx.x < 32) commit_request(c, blockIdx.x, v, view_smem + s.L, sc);
 }
 
 }  // namespace
@@ -475,15 +583,15 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream) {
 }
 
 cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream) {
-    return launch_pdl(score_kernel, dim3(a.n_req), dim3(kScoreThreads), 0, stream, a);
+    return launch_pdl(score_kernel, dim3(a.n_req), dim3(kScoreThreads), view_smem_bytes(a.L), stream, a);
 }
 
 cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream) {
-    return launch_pdl(commit_kernel, dim3(a.n_req), dim3(32), 0, stream, a);
+    return launch_pdl(commit_kernel, dim3(a.n_req), dim3(kScoreThreads), view_smem_bytes(a.L), stream, a);
 }
 
 cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStream_t stream) {
-    return launch_pdl(score_commit_kernel, dim3(s.n_req), dim3(kScoreThreads), 0, stream, s, c);
+    return launch_pdl(score_commit_kernel, dim3(s.n_req), dim3(kScoreThreads), view_smem_bytes(s.L), stream, s, c);
 }
 
 }  // namespace rps

@@ -20,10 +20,13 @@
 // own copies and stops.
 //
 // Per lane, a row segment is reduced as a base-2 online softmax against an
-// exponent reference mref that is raised only when a value exceeds it by more
-// than kSlack nats (rare):
-//   s = sum 2^u, t = sum u 2^u, u = (z - mref) log2(e)
-//   H = ln S - ln2 * T / S,  lse = mref + ln S   (after merging lanes / pieces)
+// exponent reference B (in base-2 units) that is raised only when a value exceeds
+// it by more than kSlack nats (rare):
+//   u = fma(z, log2(e), -B)  (the product is exact inside the fma),
+//   s = sum 2^u, t = sum u 2^u,
+//   H = ln S - ln2 * T / S,  lse = ln2 * B + ln S   (after merging lanes / pieces)
+// and P^max, mu and the truncated entropy take their exponents the same way, so
+// a rounding of B is a common factor of numerator and denominator.
 // The exact maximum is tracked per unit; its token index is resolved once per
 // segment by re-reading the unit that holds it.
 //
@@ -75,11 +78,6 @@ __device__ __forceinline__ f2 pack2(float lo, float hi) {
 }
 __device__ __forceinline__ void unpack2(f2 v, float &lo, float &hi) {
     asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ f2 sub2(f2 a, f2 b) {
-    f2 r;
-    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
 }
 __device__ __forceinline__ f2 mul2(f2 a, f2 b) {
     f2 r;
@@ -248,8 +246,8 @@ __device__ __forceinline__ bool j0_valid(int n_units, int lane) { return lane < 
 
 // ---------------------------------------------------------------- online softmax
 struct LaneState {
-    float mref;       // exponent reference, -inf until the first finite value
-    f2 s, t;          // pairwise partial sums of 2^u and u 2^u, u = (z - mref) log2(e)
+    float mref;       // exponent reference B (base-2 units), -inf until the first finite value
+    f2 s, t;          // pairwise partial sums of 2^u and u 2^u, u = fma(z, log2(e), -B)
     float mx;         // exact running maximum
     int best;         // unit (or first unit of the ring chunk) where mx was first reached, -1 if none
     bool best_chunk;  // best names a ring chunk: this lane's units best + 32 j, j < kBatch
@@ -270,34 +268,34 @@ __device__ __forceinline__ void lane_init(LaneState &L) {
     L.c1u = L.c2u = -1;
 }
 
-// Raise the exponent reference to m (rare: only when m exceeds it by kSlack).
+// Raise the exponent reference to m log2(e) (rare: only when m exceeds it by kSlack nats).
 __device__ __forceinline__ void raise_reference(LaneState &L, float m) {
-    if (m > L.mref + kSlack) {
+    const float mb = m * kLog2e;
+    if (mb > L.mref + kSlack * kLog2e) {
         float slo, shi;
         unpack2(L.s, slo, shi);
         if (slo + shi > 0.f) {
-            const float d = (L.mref - m) * kLog2e;
+            const float d = L.mref - mb;
             const float a = ex2(d);
             const f2 a2 = pack2(a, a);
             L.t = mul2(a2, fma2(pack2(d, d), L.s, L.t));
             L.s = mul2(a2, L.s);
         }
-        L.mref = m;
+        L.mref = mb;
     }
 }
 
-// Sums of n values (n even or the last value alone). The exponent is formed as
-// (z - mref) * log2(e): the difference is exact for values near the reference,
-// so large logits lose no absolute precision.
+// Sums of n values (n even or the last value alone). The exponent is one fma,
+// z log2(e) - B, rounded once: large logits lose no absolute precision.
 template <int N, bool SAFE>
 __device__ __forceinline__ void accumulate(LaneState &L, const float (&y)[N], int n) {
-    const f2 m2 = pack2(L.mref, L.mref);
+    const f2 m2 = pack2(-L.mref, -L.mref);
     const f2 l2 = pack2(kLog2e, kLog2e);
 #pragma unroll
     for (int i = 0; i < N; i += 2) {
         const bool v0 = i < n, v1 = i + 1 < n;
         if (!v0) break;
-        const f2 u2 = mul2(sub2(pack2(y[i], v1 ? y[i + 1] : y[i]), m2), l2);
+        const f2 u2 = fma2(pack2(y[i], v1 ? y[i + 1] : y[i]), l2, m2);
         float u0, u1;
         unpack2(u2, u0, u1);
         if (SAFE) {
@@ -642,7 +640,7 @@ __device__ __forceinline__ RowTotals combine(float mref, float s, float t, float
     r.M = warp_max(live ? mref : -INFINITY);
     float a = 0.f, d = 0.f;
     if (live) {
-        d = (mref - r.M) * kLog2e;
+        d = mref - r.M;
         a = ex2(d);
     }
     // a NaN s (bad input) must survive the merge
@@ -656,16 +654,17 @@ __device__ __forceinline__ RowTotals combine(float mref, float s, float t, float
 __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, const RowTotals &r, float tv, int ti,
                                           int lane) {
     const bool ok = (r.MX > -INFINITY) && (r.S > 0.f) && !(r.S != r.S) && !(r.T != r.T) && (r.AM != INT_MAX);
-    // Probabilities are formed relative to the exponent reference M, p_v =
-    // exp(z_v - M) / S, never as exp(z_v - lse): with large logits lse carries
-    // an absolute rounding error of ulp(lse) that the exponential would amplify.
+    // Probabilities are formed against the reference B like the sums, p_v =
+    // 2^fma(z_v, log2(e), -B) / S, never as exp(z_v - lse): with large logits
+    // lse carries an absolute rounding error of ulp(lse) that the exponential
+    // would amplify.
     float lse = NAN, H = NAN, pmax = NAN, lnS = NAN, invS = NAN;
     if (ok) {
         lnS = logf(r.S);
         invS = 1.f / r.S;
-        lse = r.M + lnS;
+        lse = fmaf(r.M, kLn2, lnS);
         H = fmaxf(lnS - kLn2 * r.T * invS, 0.f);
-        pmax = expf(r.MX - r.M) * invS;
+        pmax = ex2(fmaf(r.MX, kLog2e, -r.M)) * invS;
     }
     if (lane == 0) {
         a.zmax[slot] = ok ? r.MX : NAN;
@@ -678,9 +677,9 @@ __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, c
     if (a.k > 0) {
         float p = 0.f, h = 0.f;
         if (ok && lane < a.k) {
-            const float d = tv - r.M;  // exact for the reference's neighbourhood (Sterbenz)
-            p = expf(d) * invS;
-            if (p > 0.f) h = -p * (d - lnS);
+            const float u = fmaf(tv, kLog2e, -r.M);
+            p = ex2(u) * invS;
+            if (p > 0.f) h = -p * (u * kLn2 - lnS);
         }
         const float mu = warp_sum(p), ht = warp_sum(h);
         if (lane == 0) {
