@@ -101,6 +101,23 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
 
 
+def max_over_ranks(x: float) -> float:
+    """Largest value of x over the ranks (the slowest replica sets the job's step time)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, world: int, ms_per_step: float) -> float:
+    """Units per second of the whole job: every replica scores its own step in ms_per_step."""
+    return world * units_per_rank / (ms_per_step / 1e3)
+
+
 # ----------------------------------------------------------------------------- clocks
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -343,13 +360,9 @@ def run_gpu(args):
     with ClockSampler(local) as clk:
         step_ms, k1_ms = wl.time(args.steps, args.warmup, flush)
     clocks = clk.summary()
-    t_step = statistics.mean(step_ms)
-    if world > 1:
-        t = torch.tensor([t_step], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        t_step = float(t.item())
+    t_step = max_over_ranks(statistics.mean(step_ms))
     rows = wl.rows()
-    value = world * rows / (t_step / 1e3)
+    value = whole_job_rate(rows, world, t_step)
     k1 = statistics.mean(k1_ms)
     achieved = wl.branch_bytes() / (k1 / 1e3) / 1e9
     traffic = recorded_traffic(args.workload)
@@ -398,8 +411,8 @@ def run_gpu(args):
     if not args.skip_e2e:
         wl = Workload(w, prm, device)
         ms, h2d, d2h = wl.e2e(max(3, args.steps // 4), 2)
-        te = statistics.mean(ms)
-        out["e2e"] = {"value": world * rows / (te / 1e3), "unit": "rows/s", "h2d_bytes_per_step": h2d,
+        te = max_over_ranks(statistics.mean(ms))
+        out["e2e"] = {"value": whole_job_rate(rows, world, te), "unit": "rows/s", "h2d_bytes_per_step": h2d,
                       "d2h_bytes_per_step": d2h, "ms_per_step": te}
         del wl
         torch.cuda.empty_cache()

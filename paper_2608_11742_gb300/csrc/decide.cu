@@ -88,15 +88,6 @@ __device__ __forceinline__ uint64_t pivot_key(float v, int pos) {
     return (static_cast<uint64_t>(hi) << 32) | static_cast<uint32_t>(~pos);
 }
 
-__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const uint64_t w = __shfl_xor_sync(kFull, v, o);
-        v = w > v ? w : v;
-    }
-    return v;
-}
-
 // Dynamic shared memory of select_kernel per masked position.
 constexpr int kSelectBytesPerPos = 3 * sizeof(uint64_t) + 3 * sizeof(float) + 4 * sizeof(int32_t) + 2;
 
@@ -223,8 +214,10 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         const uint64_t *cur = keys;
         uint64_t *nxt = t_a;
         int count = n_rem;
-        for (;;) {
-            const int groups = (count + 31) / 32;
+        // P <= 16: every level at least halves count - P; 12 levels cover 4096
+        // keys, and the cap forces the last level all the same.
+        for (int level = 0;; ++level) {
+            const int groups = level == 11 ? 1 : (count + 31) / 32;
             uint64_t *dst = groups == 1 ? winners : nxt;
             const int n_dst = groups == 1 ? P : groups * P;
             for (int t = tid; t < n_dst; t += blockDim.x) dst[t] = 0ull;
@@ -232,10 +225,10 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
             for (int t = tid; t < count; t += blockDim.x) {
                 const uint64_t me = cur[t];
                 if (me == 0ull) continue;
-                const int g0 = t & ~31, g1 = min(count, g0 + 32);
+                const int g0 = groups == 1 ? 0 : t & ~31, g1 = groups == 1 ? count : min(count, g0 + 32);
                 int rank = 0;
                 for (int u = g0; u < g1; ++u) rank += cur[u] > me;
-                if (rank < P) dst[(t >> 5) * P + rank] = me;
+                if (rank < P) dst[(groups == 1 ? 0 : (t >> 5) * P) + rank] = me;
             }
             __syncthreads();
             if (groups == 1) break;
