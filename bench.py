@@ -12,9 +12,12 @@ Timing: the launches of a step are captured in one CUDA graph; each timed
 replay is preceded by an L2 flush (a 256 MB buffer is written, then read back,
 so that L2 holds none of the step's data and no dirty lines whose write-back
 would land inside the timed region) and bracketed by CUDA events on the
-launching stream; event nodes inside the graph time each kernel, including the
-lookahead row-statistics kernel (the dominant kernel), on the same stream. SM
-clocks and throttle reasons are sampled with nvidia-smi during the timed region.
+launching stream. Event nodes between kernels would break the programmatic
+dependent launch that overlaps each kernel's start with its predecessor's end,
+so the step graph has none; a second timed loop replays the same step captured
+with an event node around each kernel, on the same stream, for the per-kernel
+times and the roofline of the lookahead row-statistics kernel (the dominant
+kernel). SM clocks and throttle reasons are sampled with nvidia-smi during both.
 The roofline's `traffic` (DRAM bytes of one launch, from ncu) is reported only
 while the kernel sources hash to the value recorded beside it.
 
@@ -202,27 +205,34 @@ class Workload:
 
     def _capture(self):
         import torch
-        g = torch.cuda.CUDAGraph()
-        try:
-            ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(5)]
-        except TypeError:  # torch without external events: time the kernel in its own graph
-            ev = None
         calls = (lambda: self.step.score_base(self.logits, self.mpos, self.mcnt),
                  lambda: self.step.select(self.mpos, self.mcnt),
                  lambda: self.step.score_branch_rows(self.logits),
                  lambda: self.step.score_and_decide(self.logits))
+        g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=self.stream):
-            for i, call in enumerate(calls):
-                if ev:
-                    ev[i].record()
+            for call in calls:
                 call()
-            if ev:
+        # the same step with an event node before and after every kernel
+        self.graph_ev = torch.cuda.CUDAGraph()
+        try:
+            ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(5)]
+        except TypeError:  # torch without external events: one graph per kernel
+            ev = None
+        if ev:
+            with torch.cuda.graph(self.graph_ev, stream=self.stream):
+                for i, call in enumerate(calls):
+                    ev[i].record()
+                    call()
                 ev[4].record()
+        else:
+            self.kernel_graphs = []
+            for call in calls:
+                kg = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(kg, stream=self.stream):
+                    call()
+                self.kernel_graphs.append(kg)
         self.ev = ev
-        if ev is None:
-            self.k1_graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(self.k1_graph, stream=self.stream):
-                self.step.score_branch_rows(self.logits)
         return g
 
     def rows(self):
@@ -235,11 +245,11 @@ class Workload:
         return self.branch_rows * self.w.V * self.w.elem_bytes
 
     def time(self, steps, warmup, flush):
+        """Step times (event-free graph), then per-kernel times (graph with event nodes)."""
         import torch
         s = self.stream
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        step_ms, k1_ms = [], []
-        self.kernel_ms = {k: [] for k in self.KERNELS}
+        step_ms = []
         for i in range(warmup + steps):
             with torch.cuda.stream(s):
                 flush()
@@ -249,21 +259,28 @@ class Workload:
             s.synchronize()
             if i >= warmup:
                 step_ms.append(e0.elapsed_time(e1))
-                if self.ev:
-                    for j, name in enumerate(self.KERNELS):
-                        self.kernel_ms[name].append(self.ev[j].elapsed_time(self.ev[j + 1]))
-                    k1_ms.append(self.kernel_ms["lookahead_rows"][-1])
-        if not self.ev:
-            for i in range(warmup + steps):
+        self.kernel_ms = {k: [] for k in self.KERNELS}
+        for i in range(warmup + steps):
+            if self.ev:
                 with torch.cuda.stream(s):
                     flush()
-                    e0.record(s)
-                    self.k1_graph.replay()
-                    e1.record(s)
+                    self.graph_ev.replay()
                 s.synchronize()
                 if i >= warmup:
-                    k1_ms.append(e0.elapsed_time(e1))
-        return step_ms, k1_ms
+                    for j, name in enumerate(self.KERNELS):
+                        self.kernel_ms[name].append(self.ev[j].elapsed_time(self.ev[j + 1]))
+            else:
+                with torch.cuda.stream(s):
+                    flush()
+                for j, name in enumerate(self.KERNELS):
+                    with torch.cuda.stream(s):
+                        e0.record(s)
+                        self.kernel_graphs[j].replay()
+                        e1.record(s)
+                    s.synchronize()
+                    if i >= warmup:
+                        self.kernel_ms[name].append(e0.elapsed_time(e1))
+        return step_ms, self.kernel_ms["lookahead_rows"]
 
     def e2e(self, steps, warmup):
         """Same step through the C ABI from pinned host buffers, copies included."""
@@ -376,6 +393,8 @@ def run_gpu(args):
                               "lambda": prm.lam, "n_pivots": prm.n_pivots, "tokens_per_pivot": prm.tokens_per_pivot},
                    "rows_per_step": rows, "base_rows": wl.base_rows, "lookahead_rows": wl.branch_rows,
                    "bytes_per_step": wl.bytes(), "l2": "flushed before every timed step (256 MB buffer written, then read back)",
+                   "timing": "step: CUDA events around an event-free graph of the step; per-kernel and roofline: a "
+                             "second timed loop of the same step graph with an event node around each kernel",
                    "parallelism": f"{world} independent replica(s), no collective"},
         "achieved_gbs": wl.bytes() / (t_step / 1e3) / 1e9,
         "frac_of_hbm_peak": wl.bytes() / (t_step / 1e3) / 1e9 / peak,

@@ -956,20 +956,27 @@ __global__ void __launch_bounds__(kRowThreads, 4) row_stats_kernel(const RowStat
                 if (L.bad) L.s = pack2(NAN, NAN);
             }
         }
-        const float MX = warp_max(L.mx);
-        const int am = resolve_argmax<DT>(s.row, V, L, MX, lane);
         float tv = -INFINITY;
         int ti = INT_MAX;
+        float seg_mx = L.mx;
+        int am;
         if (TOPK) {
             // the k-th largest lane maximum bounds the segment's k-th largest logit from below
             topk_from_sketch<DT>(L, s.row, sketch, s.u0, cend, a.k, lane, warp_kth_largest(L.mx, a.k, lane), tv, ti,
                                  stage, cand);
             if (s.u1 > full_units) topk_tail<DT>(s.row, V, a.k, lane, tv, ti);
+            // rank 0 of T (largest logit, lowest token) is the argmax
+            const float t0 = __shfl_sync(kFull, tv, 0);
+            const int i0 = __shfl_sync(kFull, ti, 0);
+            seg_mx = lane == 0 ? t0 : -INFINITY;
+            am = lane == 0 ? i0 : INT_MAX;
+        } else {
+            am = resolve_argmax<DT>(s.row, V, L, warp_max(L.mx), lane);
         }
         float s_lo, s_hi, t_lo, t_hi;
         unpack2(L.s, s_lo, s_hi);
         unpack2(L.t, t_lo, t_hi);
-        RowTotals rt = combine(L.mref, s_lo + s_hi, t_lo + t_hi, L.mx, am);
+        RowTotals rt = combine(L.mref, s_lo + s_hi, t_lo + t_hi, seg_mx, am);
 
         const int64_t w_first = (r * nv) / piece;
         const int64_t w_last = ((r + 1) * nv - 1) / piece;
