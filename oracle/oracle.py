@@ -76,8 +76,8 @@ class Oracle:
                                            C.c_void_p, C.c_void_p]
         L.rps_oracle_select_pivots.restype = None
         L.rps_oracle_select_pivots.argtypes = (
-            [C.c_int32, C.c_int32, _i32p, _i32p, _f64p, _f64p, _i32p, _f64p, _f64p, _i32p, _f64p, C.c_int32,
-             C.c_double, C.c_double, C.c_double, C.c_int32, C.c_int32]
+            [C.c_int32, C.c_int32, _i32p, _i32p, _f64p, _f64p, _i32p, _f64p, _f64p, _f64p, _i32p, _f64p,
+             C.c_int32, C.c_double, C.c_double, C.c_double, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32]
             + [_i32p] * 11 + [_u8p, _i32p, _i32p, _i32p, _i32p])
         L.rps_oracle_score_branches.restype = None
         L.rps_oracle_score_branches.argtypes = (
@@ -133,9 +133,9 @@ class Oracle:
         tl = np.ascontiguousarray(base.topk_logit[:, :k_max], dtype=np.float64)
         self.lib.rps_oracle_select_pivots(
             n_req, L, np.ascontiguousarray(mask_pos, np.int32), np.ascontiguousarray(mask_cnt, np.int32),
-            base.zmax, base.pmax, base.argmax, base.mu, base.htrunc, ti, tl, k_max,
+            base.zmax, base.pmax, base.argmax, base.mu, base.htrunc, base.H, ti, tl, k_max,
             float(np.float32(params.r)), float(np.float32(params.tau_pivot)), float(np.float32(params.tau)),
-            P, K,
+            P, K, getattr(params, "commit_rule", 0), getattr(params, "commit_k", 0), getattr(params, "pivot_rule", 0),
             out["n_commit"], out["commit_pos"], out["commit_tok"], out["rem_cnt"], out["rem_k"],
             out["rem_pos"], out["state"], out["pivot_k"], out["pivot_pos"], out["n_cand"], out["cand_tok"],
             out["branch_valid"], out["branch_off"], out["branch_cnt"], out["n_branch_rows"],

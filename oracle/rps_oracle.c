@@ -46,6 +46,11 @@ enum {
     STATE_NO_CANDIDATES = 3  /* every pivot has at most one non-[MASK] candidate */
 };
 
+/* Rules for the commit set S (Eq. 2) and for the pivots (Eq. 3 and the
+ * ablation strategies of Sec. 4.3). */
+enum { COMMIT_THRESHOLD = 0, COMMIT_TOPK_CONFIDENCE = 1, COMMIT_TOPK_LOW_ENTROPY = 2 };
+enum { PIVOT_TRUNCATED_ENTROPY = 0, PIVOT_MAX_CONFIDENCE = 1, PIVOT_MAX_ENTROPY = 2 };
+
 /* Winner codes of the commit decision (>= 0: lookahead branch index b). */
 enum { WIN_ANCHOR = -1, WIN_SKIP = -2, WIN_DONE = -3 };
 
@@ -186,9 +191,10 @@ int64_t rps_oracle_row_stats(const void *logits, int32_t dtype, int64_t V,
 void rps_oracle_select_pivots(
     int32_t n_req, int32_t L, const int32_t *mask_pos, const int32_t *mask_cnt,
     const double *zmax, const double *pmax, const int32_t *argmax,
-    const double *mu, const double *htrunc,
+    const double *mu, const double *htrunc, const double *H,
     const int32_t *topk_idx, const double *topk_logit, int32_t k_max,
     double r, double tau_pivot, double tau, int32_t P, int32_t K,
+    int32_t commit_rule, int32_t commit_k, int32_t pivot_rule,
     int32_t *n_commit, int32_t *commit_pos, int32_t *commit_tok,
     int32_t *rem_cnt, int32_t *rem_k, int32_t *rem_pos, int32_t *state,
     int32_t *pivot_k, int32_t *pivot_pos, int32_t *n_cand, int32_t *cand_tok,
@@ -219,19 +225,40 @@ void rps_oracle_select_pivots(
         }
         if (cnt == 0) { state[q] = STATE_DONE; continue; }
 
-        /* Step 1: confidence-aware commit set with its fallback. */
-        int any = 0;
-        for (int32_t k = 0; k < cnt; ++k) {
-            in_S[k] = pmax[base + k] >= tau;
-            any |= in_S[k];
-        }
-        if (!any) {
-            int32_t best = 0;
-            for (int32_t k = 1; k < cnt; ++k) {
-                double a = pmax[base + k], b = pmax[base + best];
-                if (a > b || (a == b && mask_pos[base + k] < mask_pos[base + best])) best = k;
+        /* Step 1: the commit set S (Eq. 2). */
+        if (commit_rule == COMMIT_THRESHOLD) {
+            /* confidence-aware rule, with the fallback of Algorithm 1 */
+            int any = 0;
+            for (int32_t k = 0; k < cnt; ++k) {
+                in_S[k] = pmax[base + k] >= tau;
+                any |= in_S[k];
             }
-            in_S[best] = 1;
+            if (!any) {
+                int32_t best = 0;
+                for (int32_t k = 1; k < cnt; ++k) {
+                    double a = pmax[base + k], b = pmax[base + best];
+                    if (a > b || (a == b && mask_pos[base + k] < mask_pos[base + best])) best = k;
+                }
+                in_S[best] = 1;
+            }
+        } else {
+            /* top-k rules: the commit_k rows of largest P^max, or of smallest H,
+             * lower position on ties; NaN statistics rank as -inf */
+            for (int32_t k = 0; k < cnt; ++k) in_S[k] = 0;
+            for (int32_t m = 0; m < commit_k && m < cnt; ++m) {
+                int32_t best = -1;
+                double bv = 0.0;
+                for (int32_t k = 0; k < cnt; ++k) {
+                    if (in_S[k]) continue;
+                    double v = commit_rule == COMMIT_TOPK_CONFIDENCE ? pmax[base + k] : -H[base + k];
+                    if (v != v) v = -INFINITY;
+                    if (best < 0 || v > bv || (v == bv && mask_pos[base + k] < mask_pos[base + best])) {
+                        best = k;
+                        bv = v;
+                    }
+                }
+                in_S[best] = 1;
+            }
         }
         for (int32_t k = 0; k < cnt; ++k) {
             if (in_S[k]) {
@@ -248,23 +275,42 @@ void rps_oracle_select_pivots(
         /* Step 2: nothing left to search. */
         if (rem_cnt[q] == 0) { state[q] = STATE_DONE; continue; }
 
-        /* Step 3: probability-mass constraint. */
+        /* Step 3: the rows a pivot may come from. Eq. 3: the probability-mass
+         * constraint; the ablation strategies take every row of M' (NaN
+         * statistics excepted). */
         int n_feasible = 0;
         for (int32_t i = 0; i < rem_cnt[q]; ++i) {
+            const int32_t k = rem_k[base + i];
             taken[i] = 0;
-            if (mu[base + rem_k[base + i]] >= tau_pivot) n_feasible++;
+            if (pivot_rule == PIVOT_TRUNCATED_ENTROPY) {
+                if (mu[base + k] >= tau_pivot) n_feasible++;
+            } else {
+                const double v = pivot_rule == PIVOT_MAX_CONFIDENCE ? pmax[base + k] : H[base + k];
+                if (v == v) n_feasible++;
+            }
         }
         if (n_feasible == 0) { state[q] = STATE_NO_FEASIBLE; continue; }
 
-        /* Step 4: pivots by truncated entropy. */
+        /* Step 4: pivots, the P best feasible rows: by truncated entropy (Eq. 3),
+         * by confidence or by entropy; lower position on ties. */
         for (int32_t j = 0; j < P; ++j) {
             int32_t best = -1;
+            double bv = 0.0;
             for (int32_t i = 0; i < rem_cnt[q]; ++i) {
                 int32_t k = rem_k[base + i];
-                if (taken[i] || !(mu[base + k] >= tau_pivot)) continue;
-                if (best < 0) { best = i; continue; }
-                double a = htrunc[base + k], b = htrunc[base + rem_k[base + best]];
-                if (a > b || (a == b && rem_pos[base + i] < rem_pos[base + best])) best = i;
+                if (taken[i]) continue;
+                double v;
+                if (pivot_rule == PIVOT_TRUNCATED_ENTROPY) {
+                    if (!(mu[base + k] >= tau_pivot)) continue;
+                    v = htrunc[base + k];
+                } else {
+                    v = pivot_rule == PIVOT_MAX_CONFIDENCE ? pmax[base + k] : H[base + k];
+                    if (v != v) continue;
+                }
+                if (best < 0 || v > bv || (v == bv && rem_pos[base + i] < rem_pos[base + best])) {
+                    best = i;
+                    bv = v;
+                }
             }
             if (best < 0) break;
             taken[best] = 1;

@@ -31,6 +31,11 @@ class Params:
     lam: float = 0.1           # plausibility weight lambda, Eq. 4
     n_pivots: int = 4          # pivot slots P per step
     tokens_per_pivot: int = 2  # candidate tokens K per pivot
+    pivot_rule: int = 0        # 0: truncated entropy under the mass constraint (Eq. 3);
+                               # 1: max confidence, 2: max entropy (ablation strategies, Sec. 4.3)
+    commit_rule: int = 0       # 0: confidence threshold tau (Eq. 2, third rule, with the fallback);
+                               # 1: top-k confidence, 2: top-k lowest entropy (Eq. 2, first two rules)
+    commit_k: int = 0          # k of the top-k commit rules
 
     @property
     def n_branch(self) -> int:
@@ -76,7 +81,7 @@ class Workload:
 
     def params(self, base: Params = EXERCISE) -> Params:
         return Params(base.k_max, base.r, base.tau_pivot, base.tau, base.lam,
-                      self.n_pivots, self.tokens_per_pivot)
+                      self.n_pivots, self.tokens_per_pivot, base.pivot_rule, base.commit_rule, base.commit_k)
 
     def mask_counts(self) -> np.ndarray:
         if self.ragged is not None:

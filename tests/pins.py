@@ -249,9 +249,14 @@ def brute_select(logits, mask_pos, mask_cnt, prm: Params):
         if not M:
             out.append(dict(state=1, commit=[], rem=[], pivots=[], cands=[]))
             continue
-        S = [i for i in M if probs[i].max() >= np.float32(prm.tau)]
-        if not S:
-            S = [max(M, key=lambda i: (probs[i].max(), -i))]
+        if prm.commit_rule == 0:  # confidence threshold with the fallback (Eq. 2, Algorithm 1)
+            S = [i for i in M if probs[i].max() >= np.float32(prm.tau)]
+            if not S:
+                S = [max(M, key=lambda i: (probs[i].max(), -i))]
+        elif prm.commit_rule == 1:  # top-k confidence (Eq. 2, first rule)
+            S = sorted(M, key=lambda i: (-probs[i].max(), i))[:prm.commit_k]
+        else:  # top-k lowest entropy (Eq. 2, second rule)
+            S = sorted(M, key=lambda i: (_entropy64(probs[i]), i))[:prm.commit_k]
         commit = [(i, int(np.argmax(logits[q, 0, i]))) for i in M if i in S]
         rem = [i for i in M if i not in S]
         if not rem:
@@ -266,11 +271,17 @@ def brute_select(logits, mask_pos, mask_cnt, prm: Params):
         # -sum p log p over T_i only (probabilities not renormalised)
         ht = {i: float(-sum(probs[i][v] * math.log(probs[i][v]) for v in top(i) if probs[i][v] > 0))
               for i in rem}
-        feas = [i for i in rem if mu[i] >= np.float32(prm.tau_pivot)]
+        if prm.pivot_rule == 0:  # Eq. 3: mass constraint, then truncated entropy
+            feas = [i for i in rem if mu[i] >= np.float32(prm.tau_pivot)]
+            key = lambda i: (-ht[i], i)
+        elif prm.pivot_rule == 1:  # max confidence over M'
+            feas, key = list(rem), lambda i: (-probs[i].max(), i)
+        else:  # max entropy over M', unconstrained
+            feas, key = list(rem), lambda i: (-_entropy64(probs[i]), i)
         if not feas:
             out.append(dict(state=2, commit=commit, rem=rem, pivots=[], cands=[]))
             continue
-        ranked = sorted(feas, key=lambda i: (-ht[i], i))
+        ranked = sorted(feas, key=key)
         pivots = ranked[:prm.n_pivots]
         cands = []
         for i in pivots:
@@ -298,13 +309,19 @@ def _tiny_case(rng, n_req, L, V, spread):
 
 
 def pin_select_brute_force(o):
-    """Commit set, fallback, feasibility, pivots and candidates match enumeration."""
+    """Commit set, fallback, feasibility, pivots and candidates match enumeration,
+    for the paper's rules (Eq. 2 threshold, Eq. 3) and for the other commit rules
+    of Eq. 2 and the ablation pivot strategies."""
     rng = np.random.default_rng(5)
-    grid = [Params(k_max=k, r=r, tau_pivot=tp, tau=tau, lam=0.2, n_pivots=P, tokens_per_pivot=K)
-            for (k, r, tp, tau, P, K) in [
-                (4, 0.1, 0.0, 0.9, 1, 2), (4, 0.3, 0.5, 0.5, 2, 2), (6, 0.05, 0.9, 0.9, 3, 3),
-                (3, 0.5, 0.3, 0.3, 2, 1), (5, 0.2, 0.6, 0.7, 1, 5), (4, 0.1, 0.2, 0.99, 4, 2)]]
-    for trial in range(40):
+    grid = [Params(k_max=k, r=r, tau_pivot=tp, tau=tau, lam=0.2, n_pivots=P, tokens_per_pivot=K, pivot_rule=pr,
+                   commit_rule=cr, commit_k=ck)
+            for (k, r, tp, tau, P, K, pr, cr, ck) in [
+                (4, 0.1, 0.0, 0.9, 1, 2, 0, 0, 0), (4, 0.3, 0.5, 0.5, 2, 2, 0, 0, 0), (6, 0.05, 0.9, 0.9, 3, 3, 0, 0, 0),
+                (3, 0.5, 0.3, 0.3, 2, 1, 0, 0, 0), (5, 0.2, 0.6, 0.7, 1, 5, 0, 0, 0), (4, 0.1, 0.2, 0.99, 4, 2, 0, 0, 0),
+                (4, 0.1, 0.9, 0.9, 2, 2, 1, 0, 0), (4, 0.1, 0.9, 0.9, 3, 2, 2, 0, 0),
+                (4, 0.2, 0.3, 0.9, 2, 2, 0, 1, 2), (4, 0.2, 0.3, 0.9, 2, 2, 0, 2, 3),
+                (5, 0.1, 0.0, 0.5, 2, 3, 2, 1, 1), (5, 0.1, 0.0, 0.5, 3, 2, 1, 2, 4)]]
+    for trial in range(72):
         prm = grid[trial % len(grid)]
         n_req, L, V = 2, 7, 12
         z = _tiny_case(rng, n_req, L, V, rng.uniform(0.3, 2.0))

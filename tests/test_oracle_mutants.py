@@ -31,13 +31,23 @@ MUTANTS = [
      "if (a < b || (a == b && mask_pos[base + k] < mask_pos[base + best])) best = k;"),
     ("fallback tie to higher", "if (a > b || (a == b && mask_pos[base + k] < mask_pos[base + best])) best = k;",
      "if (a > b || (a == b && mask_pos[base + k] > mask_pos[base + best])) best = k;"),
-    ("feasibility strict", "if (taken[i] || !(mu[base + k] >= tau_pivot)) continue;",
-     "if (taken[i] || !(mu[base + k] > tau_pivot)) continue;"),
+    ("feasibility strict", "if (!(mu[base + k] >= tau_pivot)) continue;",
+     "if (!(mu[base + k] > tau_pivot)) continue;"),
     ("pivot by min truncated entropy",
-     "if (a > b || (a == b && rem_pos[base + i] < rem_pos[base + best])) best = i;",
-     "if (a < b || (a == b && rem_pos[base + i] < rem_pos[base + best])) best = i;"),
-    ("pivot tie to higher", "if (a > b || (a == b && rem_pos[base + i] < rem_pos[base + best])) best = i;",
-     "if (a > b || (a == b && rem_pos[base + i] > rem_pos[base + best])) best = i;"),
+     "if (best < 0 || v > bv || (v == bv && rem_pos[base + i] < rem_pos[base + best])) {",
+     "if (best < 0 || v < bv || (v == bv && rem_pos[base + i] < rem_pos[base + best])) {"),
+    ("pivot tie to higher", "if (best < 0 || v > bv || (v == bv && rem_pos[base + i] < rem_pos[base + best])) {",
+     "if (best < 0 || v > bv || (v == bv && rem_pos[base + i] > rem_pos[base + best])) {"),
+    ("top-k commit takes the smallest",
+     "if (best < 0 || v > bv || (v == bv && mask_pos[base + k] < mask_pos[base + best])) {",
+     "if (best < 0 || v < bv || (v == bv && mask_pos[base + k] < mask_pos[base + best])) {"),
+    ("lowest-entropy commit takes the highest", "pmax[base + k] : -H[base + k];", "pmax[base + k] : H[base + k];"),
+    ("max-entropy pivot uses truncated entropy",
+     "v = pivot_rule == PIVOT_MAX_CONFIDENCE ? pmax[base + k] : H[base + k];\n                    if (v != v) continue;",
+     "v = pivot_rule == PIVOT_MAX_CONFIDENCE ? pmax[base + k] : htrunc[base + k];\n                    if (v != v) continue;"),
+    ("max-confidence pivot keeps the mass constraint",
+     "v = pivot_rule == PIVOT_MAX_CONFIDENCE ? pmax[base + k] : H[base + k];\n                    if (v != v) continue;",
+     "v = pivot_rule == PIVOT_MAX_CONFIDENCE ? pmax[base + k] : H[base + k];\n                    if (v != v || !(mu[base + k] >= tau_pivot)) continue;"),
     ("candidate test absolute", "if (zt - zmax[base + k] >= log_r)", "if (zt >= log_r)"),
     ("candidate test strict", "if (zt - zmax[base + k] >= log_r)", "if (zt - zmax[base + k] > log_r)"),
     ("one candidate suffices", "if (nc >= 2) searchable = 1;", "if (nc >= 1) searchable = 1;"),
