@@ -85,8 +85,18 @@ typedef enum {
 #define RPS_WIN_SKIP (-2)   /* search skipped: the next step needs a fresh forward pass */
 #define RPS_WIN_DONE (-3)   /* nothing left to decode in this block */
 
+/* Commit-set rules (Eq. 2) and pivot rules (Eq. 3; the pivot strategies the
+ * paper's ablation compares, Sec. 4.3). */
+#define RPS_COMMIT_THRESHOLD 0        /* S = {i : P^max_i >= tau}, else the most confident row */
+#define RPS_COMMIT_TOPK_CONFIDENCE 1  /* S = the commit_k rows of largest P^max */
+#define RPS_COMMIT_TOPK_LOW_ENTROPY 2 /* S = the commit_k rows of smallest H */
+#define RPS_PIVOT_TRUNCATED_ENTROPY 0 /* Eq. 3: largest truncated entropy among mu_i >= tau_pivot */
+#define RPS_PIVOT_MAX_CONFIDENCE 1    /* largest P^max in M', no mass constraint */
+#define RPS_PIVOT_MAX_ENTROPY 2       /* largest H in M', no mass constraint */
+
 /* Limits of this build. */
 #define RPS_MAX_K 32        /* k_max */
+#define RPS_MAX_COMMIT_K 16 /* commit_k of the top-k commit rules */
 #define RPS_MAX_PIVOTS 16   /* P */
 #define RPS_MAX_POS 4096    /* L */
 #define RPS_MAX_SEGMENTS 1024
@@ -101,6 +111,9 @@ typedef struct {
     float lambda;             /* plausibility weight of Eq. 4, >= 0 */
     int32_t n_pivots;         /* P: pivot slots scored side by side, 1..RPS_MAX_PIVOTS */
     int32_t tokens_per_pivot; /* K: candidate tokens per pivot, 1..k_max */
+    int32_t pivot_rule;       /* RPS_PIVOT_*; 0 is the paper's rule */
+    int32_t commit_rule;      /* RPS_COMMIT_*; 0 is the paper's rule */
+    int32_t commit_k;         /* k of the top-k commit rules, 1..RPS_MAX_COMMIT_K (ignored by rule 0) */
 } rps_params;
 
 /* A logit tensor [n_req][n_branch][n_pos][vocab] in device memory. The vocab
@@ -215,9 +228,13 @@ rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, co
  * masked rows in mask order ([q * L + k], k < mask_cnt[q]); mask_pos lists
  * distinct positions. Per request:
  *   S = {i in M : pmax_i >= tau}, or the single most confident row (lowest
- *   position on ties) when that is empty; S is committed to argmax tokens.
+ *   position on ties) when that is empty (RPS_COMMIT_THRESHOLD); or the
+ *   commit_k rows of largest pmax / smallest H (the other rules of Eq. 2,
+ *   lower position on ties, NaN statistics last); S is committed to argmax tokens.
  *   M' = M \ S. Feasible rows: mu_i >= tau_pivot. Pivots: up to P feasible
- *   rows by truncated entropy (descending, lower position on ties).
+ *   rows by truncated entropy (descending, lower position on ties); with
+ *   RPS_PIVOT_MAX_CONFIDENCE / _MAX_ENTROPY every row of M' is feasible and
+ *   pivots are taken by pmax / H instead.
  *   Candidates: tokens of T_{i*} with z_v - zmax >= log r (that is
  *   p(v) >= r P^max), in rank order, at most K; a pivot is searched when it has
  *   at least two. Branch b = j * K + c lists M' without pivot j.

@@ -60,6 +60,12 @@ rps_status check_params(const rps_params *p, bool need_search) {
     if (!finite(p->lambda) || p->lambda < 0.f) return RPS_ERR_INVALID_ARG;
     if (p->n_pivots < 1 || p->tokens_per_pivot < 1 || p->tokens_per_pivot > p->k_max) return RPS_ERR_INVALID_ARG;
     if (p->n_pivots > RPS_MAX_PIVOTS) return RPS_ERR_UNSUPPORTED;
+    if (p->pivot_rule < RPS_PIVOT_TRUNCATED_ENTROPY || p->pivot_rule > RPS_PIVOT_MAX_ENTROPY) return RPS_ERR_INVALID_ARG;
+    if (p->commit_rule < RPS_COMMIT_THRESHOLD || p->commit_rule > RPS_COMMIT_TOPK_LOW_ENTROPY) return RPS_ERR_INVALID_ARG;
+    if (p->commit_rule != RPS_COMMIT_THRESHOLD) {
+        if (p->commit_k < 1) return RPS_ERR_INVALID_ARG;
+        if (p->commit_k > RPS_MAX_COMMIT_K) return RPS_ERR_UNSUPPORTED;
+    }
     return RPS_OK;
 }
 
@@ -184,8 +190,8 @@ rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L
                              rps_stream_t stream) {
     rps_status st = check_params(prm, true);
     if (st != RPS_OK) return st;
-    if (!base || !base->zmax || !base->pmax || !base->argmax || !base->mu || !base->htrunc || !base->topk_idx ||
-        !base->topk_logit)
+    if (!base || !base->zmax || !base->pmax || !base->argmax || !base->mu || !base->htrunc || !base->H ||
+        !base->topk_idx || !base->topk_logit)
         return RPS_ERR_INVALID_ARG;
     if (n_req < 1 || L < 1 || !d_mask_pos || !d_mask_cnt) return RPS_ERR_INVALID_ARG;
     if (L > RPS_MAX_POS) return RPS_ERR_UNSUPPORTED;
@@ -200,6 +206,7 @@ rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L
     a.pmax = base->pmax;
     a.mu = base->mu;
     a.htrunc = base->htrunc;
+    a.H = base->H;
     a.topk_logit = base->topk_logit;
     a.argmax = base->argmax;
     a.topk_idx = base->topk_idx;
@@ -213,6 +220,9 @@ rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L
     a.tau = prm->tau;
     a.tau_pivot = prm->tau_pivot;
     a.log_r = std::log(static_cast<double>(prm->r));
+    a.pivot_rule = prm->pivot_rule;
+    a.commit_rule = prm->commit_rule;
+    a.commit_k = prm->commit_k;
     a.out = *out;
     a.err = dev.err;
     return from_cuda(launch_select(a, reinterpret_cast<cudaStream_t>(stream)));
@@ -356,6 +366,6 @@ const char *rps_status_string(rps_status status) {
     return "unknown rps_status";
 }
 
-int32_t rps_version(void) { return 100; }
+int32_t rps_version(void) { return 200; }
 
 }  // extern "C"

@@ -88,8 +88,41 @@ __device__ __forceinline__ uint64_t pivot_key(float v, int pos) {
     return (static_cast<uint64_t>(hi) << 32) | static_cast<uint32_t>(~pos);
 }
 
-// Dynamic shared memory of select_kernel per masked position.
-constexpr int kSelectBytesPerPos = 3 * sizeof(uint64_t) + 3 * sizeof(float) + 4 * sizeof(int32_t) + 2;
+// The P <= RPS_MAX_PIVOTS largest of n distinct keys (0 = none), into out[0..P)
+// in descending order: in every group of 32, each key counts the larger keys of
+// its group and the best P move on, until one group is left. Every level at
+// least halves n - P, so a level's output fits t_a / t_b of n / 2 + 32 keys; the
+// level cap forces the last level all the same.
+__device__ void block_top_keys(const uint64_t *keys, int n, int P, uint64_t *t_a, uint64_t *t_b, uint64_t *out) {
+    const int tid = threadIdx.x;
+    const uint64_t *cur = keys;
+    uint64_t *nxt = t_a;
+    for (int level = 0;; ++level) {
+        const int groups = level == 11 ? 1 : (n + 31) / 32;
+        uint64_t *dst = groups <= 1 ? out : nxt;
+        const int n_dst = groups <= 1 ? P : groups * P;
+        for (int t = tid; t < n_dst; t += blockDim.x) dst[t] = 0ull;
+        __syncthreads();
+        for (int t = tid; t < n; t += blockDim.x) {
+            const uint64_t me = cur[t];
+            if (me == 0ull) continue;
+            const int g0 = groups <= 1 ? 0 : t & ~31, g1 = groups <= 1 ? n : min(n, g0 + 32);
+            int rank = 0;
+            for (int u = g0; u < g1; ++u) rank += cur[u] > me;
+            if (rank < P) dst[(groups <= 1 ? 0 : (t >> 5) * P) + rank] = me;
+        }
+        __syncthreads();
+        if (groups <= 1) return;
+        cur = nxt;
+        nxt = nxt == t_a ? t_b : t_a;
+        n = groups * P;
+    }
+}
+
+// Dynamic shared memory of select_kernel: per masked position, then a constant.
+constexpr int kSelectBytesPerPos = sizeof(uint64_t) + sizeof(uint64_t) + 4 * sizeof(float) + 4 * sizeof(int32_t) + 1;
+constexpr int kSelectBytesExtra = 2 * 32 * sizeof(uint64_t) + 16;
+__host__ __device__ constexpr int half_keys(int L) { return L / 2 + 32; }
 
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs a) {
     pdl_wait();
@@ -104,23 +137,23 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
     __shared__ Best best_buf[kSelectThreads / 32];
     __shared__ int piv_i[RPS_MAX_PIVOTS];  // index of pivot j in M'
     __shared__ int piv_nc[RPS_MAX_PIVOTS];
-    __shared__ uint64_t winners[RPS_MAX_PIVOTS];
+    __shared__ uint64_t winners[RPS_MAX_PIVOTS];  // also the commit set's keys (top-k rules)
     __shared__ int n_piv_s;
     __shared__ int br_off[RPS_MAX_PIVOTS * RPS_MAX_K + 1];
     __shared__ int16_t valid_b[RPS_MAX_PIVOTS * RPS_MAX_K];  // the m-th valid branch
     extern __shared__ __align__(16) unsigned char sel_smem[];
-    uint64_t *keys = reinterpret_cast<uint64_t *>(sel_smem);  // pivot key of M' entry i (0: infeasible)
-    uint64_t *t_a = keys + L;                           // tournament buffers
-    uint64_t *t_b = t_a + L;
-    float *pm = reinterpret_cast<float *>(t_b + L);    // P^max of mask entry k
-    float *mu = pm + L;                                // retained mass
-    float *ht = mu + L;                                // truncated entropy
-    int32_t *pos = reinterpret_cast<int32_t *>(ht + L);  // position
-    int32_t *am = pos + L;                               // argmax token
-    int32_t *rk = am + L;                                // M' entry i -> mask entry
-    int32_t *rp = rk + L;                                // M' entry i -> position
+    uint64_t *keys = reinterpret_cast<uint64_t *>(sel_smem);  // rank keys (0: none)
+    uint64_t *t_a = keys + L;                                 // tournament buffers
+    uint64_t *t_b = t_a + half_keys(L);
+    float *pm = reinterpret_cast<float *>(t_b + half_keys(L));  // P^max of mask entry k
+    float *mu = pm + L;                                         // retained mass
+    float *ht = mu + L;                                         // truncated entropy
+    float *hh = ht + L;                                         // entropy
+    int32_t *pos = reinterpret_cast<int32_t *>(hh + L);         // position
+    int32_t *am = pos + L;                                      // argmax token
+    int32_t *rk = am + L;                                       // M' entry i -> mask entry
+    int32_t *rp = rk + L;                                       // M' entry i -> position
     uint8_t *in_S = reinterpret_cast<uint8_t *>(rp + L);
-    uint8_t *taken = in_S + L;
 
     // Stage this request's statistics over the whole capacity, so that these
     // loads do not wait for the mask count (entries past it are never used),
@@ -130,6 +163,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         pm[k] = a.pmax[base + k];
         mu[k] = a.mu[base + k];
         ht[k] = a.htrunc[base + k];
+        hh[k] = a.H[base + k];
         pos[k] = a.mask_pos[base + k];
         am[k] = a.argmax[base + k];
     }
@@ -150,23 +184,42 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
     }
     __syncthreads();
 
-    // Step 1: S = {i in M : P^max_i >= tau}; fallback to the most confident row.
-    int any = 0;
-    for (int k = tid; k < cnt; k += blockDim.x) {
-        const uint8_t f = pm[k] >= a.tau;
-        in_S[k] = f;
-        any |= f;
-    }
-    any = __syncthreads_or(any);
-    if (!any && cnt > 0) {
-        Best mine{-INFINITY, INT_MAX, -1};
+    // Step 1: the commit set S (Eq. 2).
+    if (a.commit_rule == RPS_COMMIT_THRESHOLD) {
+        // S = {i in M : P^max_i >= tau}; fallback to the most confident row
+        int any = 0;
         for (int k = tid; k < cnt; k += blockDim.x) {
-            Best c{pm[k], pos[k], k};
-            if (!(c.v == c.v)) c.v = -INFINITY;  // NaN statistics never win
-            if (better(c, mine)) mine = c;
+            const uint8_t f = pm[k] >= a.tau;
+            in_S[k] = f;
+            any |= f;
         }
-        const Best b = block_best(mine, best_buf);
-        if (tid == 0) in_S[b.idx] = 1;
+        any = __syncthreads_or(any);
+        if (!any && cnt > 0) {
+            Best mine{-INFINITY, INT_MAX, -1};
+            for (int k = tid; k < cnt; k += blockDim.x) {
+                Best c{pm[k], pos[k], k};
+                if (!(c.v == c.v)) c.v = -INFINITY;  // NaN statistics never win
+                if (better(c, mine)) mine = c;
+            }
+            const Best b = block_best(mine, best_buf);
+            if (tid == 0) in_S[b.idx] = 1;
+            __syncthreads();
+        }
+    } else {
+        // S = the commit_k rows of largest P^max (or of smallest H), lower position
+        // on ties, NaN statistics last: a tournament on keys over M
+        for (int k = tid; k < cnt; k += blockDim.x) {
+            float v = a.commit_rule == RPS_COMMIT_TOPK_CONFIDENCE ? pm[k] : -hh[k];
+            if (!(v == v)) v = -INFINITY;
+            keys[k] = pivot_key(v, pos[k]);
+        }
+        __syncthreads();
+        block_top_keys(keys, cnt, a.commit_k, t_a, t_b, winners);
+        for (int k = tid; k < cnt; k += blockDim.x) {
+            uint8_t f = 0;
+            for (int j = 0; j < a.commit_k; ++j) f |= keys[k] == winners[j];
+            in_S[k] = f;
+        }
         __syncthreads();
     }
 
@@ -185,7 +238,12 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
                 const int r = k - (n_commit + excl);
                 rk[r] = k;
                 rp[r] = pos[k];
-                keys[r] = mu[k] >= a.tau_pivot && ht[k] == ht[k] ? pivot_key(ht[k], pos[k]) : 0ull;
+                if (a.pivot_rule == RPS_PIVOT_TRUNCATED_ENTROPY)
+                    keys[r] = mu[k] >= a.tau_pivot && ht[k] == ht[k] ? pivot_key(ht[k], pos[k]) : 0ull;
+                else {
+                    const float v = a.pivot_rule == RPS_PIVOT_MAX_CONFIDENCE ? pm[k] : hh[k];
+                    keys[r] = v == v ? pivot_key(v, pos[k]) : 0ull;
+                }
                 o.rem_k[base + r] = k;
                 o.rem_pos[base + r] = pos[k];
             }
@@ -202,40 +260,13 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
         if (tid == 0) o.state[q] = RPS_STATE_DONE;
         return;
     }
-    for (int i = tid; i < n_rem; i += blockDim.x) taken[i] = 0;
     __syncthreads();
 
-    // Steps 3-4: feasibility (mu >= tau_pivot) and the P best feasible rows by
-    // truncated entropy (descending, lower position on ties), as a tournament on
-    // the keys: in every group of 32, each key counts the larger keys of its group
-    // and the P best move on, until one group is left. Keys are distinct (0, the
-    // infeasible mark, excepted), so ranks are too.
+    // Steps 3-4: the P best feasible rows of M' by their key -- truncated
+    // entropy under the mass constraint (Eq. 3), or confidence, or entropy --
+    // lower position on ties, by a tournament on the keys.
     {
-        const uint64_t *cur = keys;
-        uint64_t *nxt = t_a;
-        int count = n_rem;
-        // P <= 16: every level at least halves count - P; 12 levels cover 4096
-        // keys, and the cap forces the last level all the same.
-        for (int level = 0;; ++level) {
-            const int groups = level == 11 ? 1 : (count + 31) / 32;
-            uint64_t *dst = groups == 1 ? winners : nxt;
-            const int n_dst = groups == 1 ? P : groups * P;
-            for (int t = tid; t < n_dst; t += blockDim.x) dst[t] = 0ull;
-            __syncthreads();
-            for (int t = tid; t < count; t += blockDim.x) {
-                const uint64_t me = cur[t];
-                if (me == 0ull) continue;
-                const int g0 = groups == 1 ? 0 : t & ~31, g1 = groups == 1 ? count : min(count, g0 + 32);
-                int rank = 0;
-                for (int u = g0; u < g1; ++u) rank += cur[u] > me;
-                if (rank < P) dst[(groups == 1 ? 0 : (t >> 5) * P) + rank] = me;
-            }
-            __syncthreads();
-            if (groups == 1) break;
-            cur = nxt;
-            nxt = nxt == t_a ? t_b : t_a;
-            count = groups * P;
-        }
+        block_top_keys(keys, n_rem, P, t_a, t_b, winners);
         if (tid == 0) {
             int c = 0;
             while (c < P && winners[c] != 0ull) ++c;
@@ -566,7 +597,7 @@ __global__ void __launch_bounds__(kScoreThreads) score_commit_kernel(const Score
 }  // namespace
 
 cudaError_t launch_select(const SelectArgs &a, cudaStream_t stream) {
-    const size_t smem = static_cast<size_t>(a.L) * kSelectBytesPerPos + 16;
+    const size_t smem = static_cast<size_t>(a.L) * kSelectBytesPerPos + kSelectBytesExtra;
     if (smem > 48 * 1024) {
         const cudaError_t e =
             cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));

@@ -66,13 +66,14 @@ cudaError_t row_stats_occupancy(int dtype, bool topk, int *blocks_per_sm);
 
 struct SelectArgs {
     // base statistics [q * L + k]
-    const float *zmax, *pmax, *mu, *htrunc, *topk_logit;
+    const float *zmax, *pmax, *mu, *htrunc, *H, *topk_logit;
     const int32_t *argmax, *topk_idx;
     int32_t k_max;
     const int32_t *mask_pos, *mask_cnt;
     int32_t n_req, L, P, K;
     float tau, tau_pivot;
     double log_r;
+    int32_t pivot_rule, commit_rule, commit_k;
     rps_pivots out;
     uint32_t *err;
 };

@@ -38,7 +38,8 @@ _p = C.c_void_p
 
 class RpsParams(C.Structure):
     _fields_ = [("k_max", C.c_int32), ("r", C.c_float), ("tau_pivot", C.c_float), ("tau", C.c_float),
-                ("lambda_", C.c_float), ("n_pivots", C.c_int32), ("tokens_per_pivot", C.c_int32)]
+                ("lambda_", C.c_float), ("n_pivots", C.c_int32), ("tokens_per_pivot", C.c_int32),
+                ("pivot_rule", C.c_int32), ("commit_rule", C.c_int32), ("commit_k", C.c_int32)]
 
 
 class RpsLogits(C.Structure):
@@ -129,7 +130,8 @@ def _stream(stream) -> Optional[int]:
 
 def params(p) -> RpsParams:
     """C struct from any object with the ``configs.Params`` fields."""
-    return RpsParams(p.k_max, p.r, p.tau_pivot, p.tau, p.lam, p.n_pivots, p.tokens_per_pivot)
+    return RpsParams(p.k_max, p.r, p.tau_pivot, p.tau, p.lam, p.n_pivots, p.tokens_per_pivot,
+                     getattr(p, "pivot_rule", 0), getattr(p, "commit_rule", 0), getattr(p, "commit_k", 0))
 
 
 def logits_desc(t: torch.Tensor) -> RpsLogits:

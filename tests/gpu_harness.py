@@ -75,27 +75,41 @@ def piv_np(buf: rps.PivotsBuf) -> dict:
 def near_threshold_requests(o: RowStats, piv_o: dict, mask_cnt, L, prm) -> set:
     """Requests whose selection hinges on an oracle quantity within BAND of its threshold.
 
-    Only the comparisons that decide the outcome count: P^max against tau, the
-    two most confident rows (fallback), mu against tau_pivot, and adjacent
-    truncated entropies among the P + 1 highest feasible rows of M'.
+    Only the comparisons that decide the outcome count. Commit set: P^max
+    against tau and the two most confident rows (threshold rule and its
+    fallback), or adjacent values among the k + 1 best of M (top-k rules).
+    Pivots: mu against tau_pivot and adjacent truncated entropies among the
+    P + 1 highest feasible rows of M' (Eq. 3), or adjacent confidences /
+    entropies among the P + 1 highest rows of M' (the other pivot rules).
     """
+    def close_pair(values, n):
+        v = np.sort(np.asarray(values, np.float64))[::-1][:n]
+        return len(v) > 1 and np.min(-np.diff(v)) < BAND
+
+    commit_rule = getattr(prm, "commit_rule", 0)
+    pivot_rule = getattr(prm, "pivot_rule", 0)
     out = set()
     tau, tau_p = np.float32(prm.tau), np.float32(prm.tau_pivot)
     for q in range(len(mask_cnt)):
         s = slice(q * L, q * L + int(mask_cnt[q]))
-        pm, mu = o.pmax[s], o.mu[s]
-        if np.any(np.abs(pm - tau) < BAND) or np.any(np.abs(mu - tau_p) < BAND):
-            out.add(q)
-            continue
-        if len(pm) > 1:
-            top = np.sort(pm)[::-1]
-            if top[0] - top[1] < BAND:
+        pm, mu, H = o.pmax[s], o.mu[s], o.H[s]
+        if commit_rule == 0:
+            if np.any(np.abs(pm - tau) < BAND) or close_pair(pm, 2):
                 out.add(q)
                 continue
+        elif close_pair(pm if commit_rule == 1 else -H, prm.commit_k + 1):
+            out.add(q)
+            continue
         rem = piv_o["rem_k"][q, :piv_o["rem_cnt"][q]]
-        feas = [k for k in rem if o.mu[q * L + k] >= tau_p]
-        ht = np.sort(np.array([o.htrunc[q * L + k] for k in feas]))[::-1][:prm.n_pivots + 1]
-        if len(ht) > 1 and np.min(-np.diff(ht)) < BAND:
+        if pivot_rule == 0:
+            if np.any(np.abs(np.array([o.mu[q * L + k] for k in rem]) - tau_p) < BAND):
+                out.add(q)
+                continue
+            vals = [o.htrunc[q * L + k] for k in rem if o.mu[q * L + k] >= tau_p]
+        else:
+            src = o.pmax if pivot_rule == 1 else o.H
+            vals = [src[q * L + k] for k in rem]
+        if close_pair(vals, prm.n_pivots + 1):
             out.add(q)
     return out
 

@@ -119,6 +119,10 @@ def test_host_rejects_bad_arguments(libs):
     assert select(prm=r.RpsParams(10, 0.1, 0.9, 0.9, 0.1, 17, 2)) == r.RPS_ERR_UNSUPPORTED  # P > 16
     nan = float("nan")
     assert select(prm=r.RpsParams(10, 0.1, nan, 0.9, 0.1, 4, 2)) == r.RPS_ERR_INVALID_ARG
+    assert select(prm=r.RpsParams(10, 0.1, 0.9, 0.9, 0.1, 4, 2, 3, 0, 0)) == r.RPS_ERR_INVALID_ARG  # pivot rule
+    assert select(prm=r.RpsParams(10, 0.1, 0.9, 0.9, 0.1, 4, 2, 0, 3, 1)) == r.RPS_ERR_INVALID_ARG  # commit rule
+    assert select(prm=r.RpsParams(10, 0.1, 0.9, 0.9, 0.1, 4, 2, 0, 1, 0)) == r.RPS_ERR_INVALID_ARG  # top-k, k = 0
+    assert select(prm=r.RpsParams(10, 0.1, 0.9, 0.9, 0.1, 4, 2, 0, 2, 17)) == r.RPS_ERR_UNSUPPORTED  # k > 16
     holes = r.RpsPivots(*([fake] * (len(r._PIVOT_FIELDS) - 1) + [None]))
     assert select(piv=holes) == r.RPS_ERR_INVALID_ARG
 

@@ -197,6 +197,11 @@ PARAM_MATRIX = [
     Params(k_max=32, r=0.05, tau_pivot=0.0, n_pivots=1, tokens_per_pivot=32),   # adaptive C, one pivot
     Params(k_max=5, r=0.3, tau_pivot=0.0, lam=0.2, n_pivots=8, tokens_per_pivot=3),
     Params(tau=0.05, tau_pivot=0.0, lam=5.0),                 # plausibility dominates: abstain
+    # the other commit rules of Eq. 2 and the ablation pivot strategies
+    Params(tau_pivot=0.0, pivot_rule=1),                      # max-confidence pivots
+    Params(tau_pivot=0.9, pivot_rule=2),                      # max-entropy pivots, no mass constraint
+    Params(tau_pivot=0.0, commit_rule=1, commit_k=2),         # top-k confidence commits
+    Params(tau_pivot=0.003, commit_rule=2, commit_k=3, pivot_rule=2),  # lowest-entropy commits
 ]
 
 STEP_CASES = [
