@@ -281,6 +281,28 @@ rps_status rps_score_and_commit(const rps_logits *anchor_logits, int32_t anchor_
                                 const rps_pivots *piv, const rps_params *prm, const rps_branch_scores *scores,
                                 const rps_commit_out *out, rps_stream_t stream);
 
+/*
+ * Outer loop of Algorithm 1 over semi-autoregressive blocks (the response of
+ * L_total positions is decoded block by block, B positions each, left to
+ * right). Call after rps_commit of a step whose mask arrays are block-local
+ * ([n_req][B], positions 0..B-1 of the current block). Per request:
+ *   tokens[q][b * B + p] = the token committed at block position p this step
+ *     (the standard commit S of `piv` and the pivot committed by `commit`);
+ *   the next step's mask (d_mask_pos / d_mask_cnt) is commit->mask_* while
+ *     the block has masked positions, else the whole next block (block[q]
+ *     advances), else empty with done[q] = 1.
+ * Device arrays: d_tokens [n_req][L_total] (-1 while masked, caller-initialised),
+ * d_block [n_req], d_mask_pos [n_req][B], d_mask_cnt [n_req], d_done [n_req]
+ * (in/out); d_steps [n_req] (optional, NULL to skip) counts the steps each
+ * request took before it was done. commit->mask_* may alias d_mask_*. A commit
+ * list outside the block sets RPS_DEVERR_MASK.
+ * Errors: RPS_ERR_INVALID_ARG for NULL pointers or sizes out of range;
+ * RPS_ERR_UNSUPPORTED when B > RPS_MAX_POS.
+ */
+rps_status rps_decode_advance(const rps_pivots *piv, const rps_commit_out *commit, int32_t n_req, int32_t B,
+                              int32_t L_total, int32_t *d_tokens, int32_t *d_block, int32_t *d_mask_pos,
+                              int32_t *d_mask_cnt, int32_t *d_done, int32_t *d_steps, rps_stream_t stream);
+
 /* Bytes of scratch the library holds on each device for rps_score_step_noalloc. */
 #define RPS_STATIC_SCRATCH_BYTES (8u << 20)
 

@@ -34,6 +34,29 @@ int32_t rps_synth_fill(void *out, int32_t dtype, int32_t n_req, int32_t n_branch
                        uint64_t t_low, uint64_t t_mid, uint32_t step, const float *scale, const int32_t *epoch,
                        const uint8_t *valid, void *stream);
 
+
+/*
+ * Decode mode: the current semi-autoregressive block of every request. Row p of
+ * request q is response position d_block[q] * B + p (rows past L_total are NaN);
+ * the branch factors use the step index *d_step; scale and epoch are
+ * [n_req][L_total] device arrays over the response. All pointers are device
+ * pointers. Returns as rps_synth_fill.
+ */
+int32_t rps_synth_fill_blocks(void *out, int32_t dtype, int32_t n_req, int32_t n_branch, int32_t B, int64_t vocab,
+                              int64_t req_stride, int64_t branch_stride, int64_t pos_stride, uint32_t seed,
+                              uint64_t t_low, uint64_t t_mid, const int32_t *d_step, const int32_t *d_block,
+                              int32_t L_total, const float *scale, const int32_t *epoch, void *stream);
+
+/*
+ * Apply one step's decisions (d_winner [n_req], the winner codes of rps_commit)
+ * to the generator state of each request's current block -- a committed branch b
+ * multiplies the spike scale by that branch's factor of the step, a skip (-2)
+ * advances the noise epoch -- then advance *d_step. Returns 0, 1 for invalid
+ * arguments, 2 for a CUDA launch error.
+ */
+int32_t rps_synth_advance(const int32_t *d_winner, int32_t n_req, int32_t B, int32_t L_total, const int32_t *d_block,
+                          int32_t *d_step, float *scale, int32_t *epoch, uint32_t seed, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

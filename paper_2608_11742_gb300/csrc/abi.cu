@@ -104,6 +104,12 @@ WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k
 rps_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RPS_OK : RPS_ERR_CUDA; }
 
 }  // namespace
+
+uint32_t *device_error_word() {
+    DeviceInfo dev;
+    return device_info(&dev) == RPS_OK ? dev.err : nullptr;
+}
+
 }  // namespace rps
 
 using namespace rps;

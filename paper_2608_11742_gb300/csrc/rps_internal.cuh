@@ -104,6 +104,9 @@ cudaError_t launch_score(const ScoreArgs &a, cudaStream_t stream);
 cudaError_t launch_commit(const CommitArgs &a, cudaStream_t stream);
 cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStream_t stream);
 
+// The calling device's sticky error word (nullptr if the device cannot be queried).
+uint32_t *device_error_word();
+
 // ---------------------------------------------------------------- launches
 // Every kernel of the library is launched with programmatic stream
 // serialization: it may start while the previous kernel on the stream finishes,

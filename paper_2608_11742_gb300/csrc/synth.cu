@@ -60,10 +60,24 @@ struct Args {
     const float *scale;
     const int32_t *epoch;
     const uint8_t *valid;
+    // decode mode (d_block != nullptr): row p of request q is response position
+    // d_block[q] * L + p; scale / epoch are [n_req][state_L] over the response;
+    // rows past the response end are NaN; the step index is read from d_step
+    const int32_t *d_step;
+    const int32_t *d_block;
+    int32_t state_L;
 };
+
+// Spike scale factor in [0.8, 1.6) of branch b >= 1 at (q, pos), drawn per step.
+__device__ __forceinline__ float branch_factor(uint32_t seed, int q, int b, int pos, uint32_t step) {
+    const U4 bf = philox(b, pos, q, tag(kTagBranch, step), seed, kKey1);
+    const float u = __fmul_rn(static_cast<float>(bf.x >> 8), 5.9604644775390625e-8f);
+    return __fadd_rn(0.8f, __fmul_rn(0.8f, u));
+}
 
 __global__ void fill_kernel(const Args a) {
     const int64_t V = a.vocab;
+    const uint32_t step = a.d_step ? static_cast<uint32_t>(*a.d_step) : a.step;
     const int64_t chunks = (V + kPerThread - 1) / kPerThread;
     const int64_t rows = static_cast<int64_t>(a.n_req) * (a.n_branch + 1) * a.L;
     const int64_t total = rows * chunks;
@@ -71,12 +85,15 @@ __global__ void fill_kernel(const Args a) {
          g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t row = g / chunks;
         const int64_t v0 = (g - row * chunks) * kPerThread;
-        const int pos = static_cast<int>(row % a.L);
+        const int local = static_cast<int>(row % a.L);
         const int b = static_cast<int>((row / a.L) % (a.n_branch + 1));
         const int q = static_cast<int>(row / (static_cast<int64_t>(a.L) * (a.n_branch + 1)));
-        const int64_t off = q * a.req_stride + b * a.branch_stride + pos * a.pos_stride + v0;
+        const int64_t off = q * a.req_stride + b * a.branch_stride + local * a.pos_stride + v0;
         const int n = static_cast<int>((V - v0 < kPerThread ? V - v0 : static_cast<int64_t>(kPerThread)));
-        const bool is_valid = a.valid == nullptr || a.valid[static_cast<int64_t>(q) * a.L + pos] != 0;
+        const int pos = a.d_block ? a.d_block[q] * a.L + local : local;  // position in the response
+        const bool is_valid = a.d_block ? pos < a.state_L
+                                        : a.valid == nullptr || a.valid[static_cast<int64_t>(q) * a.L + local] != 0;
+        const int64_t state_row = static_cast<int64_t>(q) * a.state_L + pos;
 
         float z[kPerThread];
         if (!is_valid) {
@@ -112,16 +129,11 @@ __global__ void fill_kernel(const Args a) {
             float amp = 0.f;
             if (regime != 2) {
                 const float h = regime == 0 ? 12.0f : 4.0f;
-                const float sc = a.scale ? a.scale[static_cast<int64_t>(q) * a.L + pos] : 1.0f;
-                float f = 1.0f;
-                if (b > 0) {
-                    const U4 bf = philox(b, pos, q, tag(kTagBranch, a.step), a.seed, kKey1);
-                    const float u = __fmul_rn(static_cast<float>(bf.x >> 8), 5.9604644775390625e-8f);
-                    f = __fadd_rn(0.8f, __fmul_rn(0.8f, u));
-                }
+                const float sc = a.scale ? a.scale[state_row] : 1.0f;
+                const float f = b > 0 ? branch_factor(a.seed, q, b, pos, step) : 1.0f;
                 amp = __fmul_rn(__fmul_rn(h, sc), f);
             }
-            const uint32_t ep = a.epoch ? static_cast<uint32_t>(a.epoch[static_cast<int64_t>(q) * a.L + pos]) : 0u;
+            const uint32_t ep = a.epoch ? static_cast<uint32_t>(a.epoch[state_row]) : 0u;
 #pragma unroll
             for (int i = 0; i < kPerThread; ++i) {
                 if (i >= n) {
@@ -192,10 +204,88 @@ extern "C" int32_t rps_synth_fill(void *out, int32_t dtype, int32_t n_req, int32
     a.scale = scale;
     a.epoch = epoch;
     a.valid = valid;
+    a.d_step = nullptr;
+    a.d_block = nullptr;
+    a.state_L = L;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (sms < 1) sms = 1;
     fill_kernel<<<sms * 8, 256, 0, static_cast<cudaStream_t>(stream)>>>(a);
+    return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+namespace {
+
+// The decision of a step applied to the generator state of the positions of
+// each request's current block: a committed branch becomes the next base (its
+// spike factor of the step multiplies the spike scale), a skip draws fresh noise
+// (the noise epoch advances), an abstain or a finished request changes nothing.
+__global__ void advance_kernel(const int32_t *winner, int32_t B, int32_t L_total, const int32_t *d_block,
+                               const int32_t *d_step, float *scale, int32_t *epoch, uint32_t seed) {
+    const int q = blockIdx.x;
+    const int w = winner[q];
+    const uint32_t step = static_cast<uint32_t>(*d_step);
+    const int base = d_block[q] * B;
+    for (int p = threadIdx.x; p < B; p += blockDim.x) {
+        const int pos = base + p;
+        if (pos >= L_total) break;
+        const int64_t i = static_cast<int64_t>(q) * L_total + pos;
+        if (w >= 0) scale[i] = __fmul_rn(scale[i], branch_factor(seed, q, 1 + w, pos, step));
+        else if (w == -2) epoch[i] += 1;
+    }
+}
+
+__global__ void step_kernel(int32_t *d_step) { *d_step += 1; }
+
+}  // namespace
+
+extern "C" int32_t rps_synth_fill_blocks(void *out, int32_t dtype, int32_t n_req, int32_t n_branch, int32_t B,
+                                         int64_t vocab, int64_t req_stride, int64_t branch_stride, int64_t pos_stride,
+                                         uint32_t seed, uint64_t t_low, uint64_t t_mid, const int32_t *d_step,
+                                         const int32_t *d_block, int32_t L_total, const float *scale,
+                                         const int32_t *epoch, void *stream) {
+    if (!out || !d_step || !d_block || !scale || !epoch || (dtype != 0 && dtype != 1) || n_req < 1 || n_branch < 0 ||
+        B < 1 || L_total < 1 || vocab < 1 || vocab > 0xFFFFFFFFLL || t_low > t_mid || t_mid > (1ull << 32))
+        return 1;
+    const int64_t esize = dtype == 1 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(out) % 16 || (req_stride * esize) % 16 || (branch_stride * esize) % 16 ||
+        (pos_stride * esize) % 16)
+        return 1;
+    Args a;
+    a.out = out;
+    a.dtype = dtype;
+    a.n_req = n_req;
+    a.n_branch = n_branch;
+    a.L = B;
+    a.vocab = vocab;
+    a.req_stride = req_stride;
+    a.branch_stride = branch_stride;
+    a.pos_stride = pos_stride;
+    a.seed = seed;
+    a.step = 0;
+    a.t_low = t_low;
+    a.t_mid = t_mid;
+    a.scale = scale;
+    a.epoch = epoch;
+    a.valid = nullptr;
+    a.d_step = d_step;
+    a.d_block = d_block;
+    a.state_L = L_total;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms < 1) sms = 1;
+    fill_kernel<<<sms * 8, 256, 0, static_cast<cudaStream_t>(stream)>>>(a);
+    return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+extern "C" int32_t rps_synth_advance(const int32_t *d_winner, int32_t n_req, int32_t B, int32_t L_total,
+                                     const int32_t *d_block, int32_t *d_step, float *scale, int32_t *epoch,
+                                     uint32_t seed, void *stream) {
+    if (!d_winner || !d_block || !d_step || !scale || !epoch || n_req < 1 || B < 1 || L_total < 1) return 1;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    advance_kernel<<<n_req, 256, 0, s>>>(d_winner, B, L_total, d_block, d_step, scale, epoch, seed);
+    step_kernel<<<1, 1, 0, s>>>(d_step);
     return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }

@@ -99,6 +99,9 @@ _lib.rps_score_and_commit.restype = C.c_int
 _lib.rps_score_and_commit.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.POINTER(RpsRowStats),
                                       C.POINTER(RpsRowStats), C.c_int32, C.c_int32, C.POINTER(RpsPivots),
                                       C.POINTER(RpsParams), C.POINTER(RpsBranchScores), C.POINTER(RpsCommitOut), _p]
+_lib.rps_decode_advance.restype = C.c_int
+_lib.rps_decode_advance.argtypes = [C.POINTER(RpsPivots), C.POINTER(RpsCommitOut), C.c_int32, C.c_int32, C.c_int32,
+                                    _p, _p, _p, _p, _p, _p, _p]
 _lib.rps_poll_device_status.restype = C.c_int
 _lib.rps_poll_device_status.argtypes = [_p, C.POINTER(C.c_uint32)]
 _lib.rps_status_string.restype = C.c_char_p
@@ -317,6 +320,15 @@ def rps_score_and_commit(anchor_logits: torch.Tensor, anchor_branch: int, anchor
     s, o = scores.c(), out.c()
     _check(_lib.rps_score_and_commit(C.byref(d), anchor_branch, C.byref(a), C.byref(b), n_req, L, C.byref(pv),
                                      C.byref(p), C.byref(s), C.byref(o), _stream(stream)), "rps_score_and_commit")
+
+
+def rps_decode_advance(piv: PivotsBuf, commit: CommitBuf, n_req: int, B: int, L_total: int, tokens, block, mask_pos,
+                       mask_cnt, done, steps=None, stream=None) -> None:
+    pv, cm = piv.c(), commit.c()
+    _check(_lib.rps_decode_advance(C.byref(pv), C.byref(cm), n_req, B, L_total, tokens.data_ptr(), block.data_ptr(),
+                                   mask_pos.data_ptr(), mask_cnt.data_ptr(), done.data_ptr(),
+                                   None if steps is None else steps.data_ptr(), _stream(stream)),
+           "rps_decode_advance")
 
 
 def rps_poll_device_status(stream=None):

@@ -254,6 +254,13 @@ def _synth_lib():
         lib.rps_synth_fill.argtypes = [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int64,
                                        C.c_int64, C.c_int64, C.c_int64, C.c_uint32, C.c_uint64, C.c_uint64,
                                        C.c_uint32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
+        lib.rps_synth_fill_blocks.restype = C.c_int32
+        lib.rps_synth_fill_blocks.argtypes = [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int64,
+                                              C.c_int64, C.c_int64, C.c_int64, C.c_uint32, C.c_uint64, C.c_uint64,
+                                              C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]
+        lib.rps_synth_advance.restype = C.c_int32
+        lib.rps_synth_advance.argtypes = [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
+                                          C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]
         _SYNTH_LIB = lib
     return _SYNTH_LIB
 
@@ -278,3 +285,34 @@ def device_fill(out, seed: int, mixture, step: int = 0, scale=None, epoch=None, 
                                      stream.cuda_stream)
     if rc != 0:
         raise RuntimeError(f"rps_synth_fill failed with code {rc}")
+
+
+def device_fill_blocks(out, seed: int, mixture, d_step, d_block, L_total: int, scale, epoch, stream=None) -> None:
+    """Decode mode of ``device_fill``: ``out`` is ``[n_req][1 + n_branch][B][V]``, the
+    current block of every request (row p is response position ``d_block[q] * B + p``;
+    rows past ``L_total`` are NaN). ``d_step`` (int32 [1]), ``d_block`` (int32 [n_req]),
+    ``scale`` (float32) and ``epoch`` (int32) ``[n_req][L_total]`` are CUDA tensors."""
+    import torch
+    dtype = {torch.bfloat16: 1, torch.float32: 0}[out.dtype]
+    n_req, nb1, B, V = out.shape
+    t_low, t_mid = regime_thresholds(mixture)
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    rc = _synth_lib().rps_synth_fill_blocks(out.data_ptr(), dtype, n_req, nb1 - 1, B, V, out.stride(0), out.stride(1),
+                                            out.stride(2), seed, t_low, t_mid, d_step.data_ptr(), d_block.data_ptr(),
+                                            L_total, scale.data_ptr(), epoch.data_ptr(), stream.cuda_stream)
+    if rc != 0:
+        raise RuntimeError(f"rps_synth_fill_blocks failed with code {rc}")
+
+
+def device_advance(winner, B: int, L_total: int, d_block, d_step, scale, epoch, seed: int, stream=None) -> None:
+    """Apply one step's winner codes to the generator state of each current block,
+    then advance the step counter (all CUDA tensors; see ``rps_synth_advance``)."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    rc = _synth_lib().rps_synth_advance(winner.data_ptr(), winner.shape[0], B, L_total, d_block.data_ptr(),
+                                        d_step.data_ptr(), scale.data_ptr(), epoch.data_ptr(), seed,
+                                        stream.cuda_stream)
+    if rc != 0:
+        raise RuntimeError(f"rps_synth_advance failed with code {rc}")
