@@ -316,6 +316,34 @@ class Workload:
         return ms, h2d, d2h
 
 
+def decode_run(configs, device):
+    """A whole response decoded on the device (Algorithm 1): the block workload's
+    64 requests x 32-position blocks extended to 256 positions. The denoiser
+    forward pass is the seeded generator (a stub); its time is reported apart."""
+    import torch
+    from paper_2608_11742_gb300.decode import DecodeLoop
+    w = configs.BLOCK
+    prm = w.params(configs.EXERCISE)
+    L_total = 256
+    loop = DecodeLoop(w.n_req, w.L, L_total, w.V, prm, w.seed, w.mixture, device)
+    stream = torch.cuda.Stream(device)
+    steps, score_ms, total_ms = loop.run_split(stream)
+    rows = int(loop.steps.sum().item())  # request-steps
+    tokens = w.n_req * L_total
+    mean_ms = statistics.mean(score_ms)
+    return {"workload": f"{w.n_req} requests x {L_total} positions in blocks of {w.L}, vocab {w.V}, bf16, "
+                        f"1 base + {w.n_branch} lookahead branches, mixture {w.mixture}",
+            "decoded": bool(loop.done.all().item()) and bool((loop.tokens >= 0).all().item()),
+            "steps": steps, "request_steps": rows, "tokens": tokens,
+            "scoring_ms_per_step": mean_ms, "scoring_p50_ms": statistics.median(score_ms),
+            "tokens_per_s_scoring": tokens / (sum(score_ms) / 1e3),
+            "total_ms_with_stub": total_ms,
+            "launches_per_step": DecodeLoop.LAUNCHES,
+            "timing": "CUDA events around the graph of the scoring step (row statistics, selection, lookahead "
+                      "rows, scores and commit, decode advance), replayed after the stub's graph wrote the step's "
+                      "4.66 GB of logits (larger than L2)"}
+
+
 def cpu_sample(w, n_take: int = 64):
     """A bounded sample of one step's rows, in the step's proportions: base rows
     (scored in top-k mode) and lookahead rows (statistics only)."""
@@ -427,6 +455,10 @@ def run_gpu(args):
             torch.cuda.empty_cache()
         out["other_workloads"] = others
 
+    if not args.skip_decode:
+        out["decode"] = decode_run(configs, device)
+        torch.cuda.empty_cache()
+
     if not args.skip_e2e:
         wl = Workload(w, prm, device)
         ms, h2d, d2h = wl.e2e(max(3, args.steps // 4), 2)
@@ -484,6 +516,7 @@ def main():
     ap.add_argument("--workload", default=HEADLINE)
     ap.add_argument("--skip-others", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--skip-decode", action="store_true")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()

@@ -89,6 +89,44 @@ class DecodeLoop:
         self.d_step.zero_()
         self.steps.zero_()
 
+    def run_split(self, stream, check_every: int = 8):
+        """Decode to the end with the forward stub and the scoring step captured as
+        two graphs, timing each scoring replay with CUDA events on ``stream``.
+        Returns (steps, per-step scoring ms, total ms)."""
+        with torch.cuda.stream(stream):
+            self.step_once(stream)
+        stream.synchronize()
+        self.reset()
+        g_fwd, g_score = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_fwd, stream=stream):
+            self.forward_stub(stream)
+        with torch.cuda.graph(g_score, stream=stream):
+            self.score_and_advance(stream)
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev = []
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+        steps = 0
+        while steps < self.L_total:
+            for _ in range(check_every):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                with torch.cuda.stream(stream):
+                    g_fwd.replay()
+                    e0.record(stream)
+                    g_score.replay()
+                    e1.record(stream)
+                ev.append((e0, e1))
+            steps += check_every
+            stream.synchronize()
+            if bool(self.done.all()):
+                break
+        with torch.cuda.stream(stream):
+            t1.record(stream)
+        stream.synchronize()
+        taken = int(self.steps.max().item())
+        score_ms = [a.elapsed_time(b) for a, b in ev[:taken]]
+        return taken, score_ms, t0.elapsed_time(t1)
+
     def run(self, stream, max_steps: int | None = None, check_every: int = 16) -> int:
         """Replay the step graph until every request is done; returns the steps taken.
         Each step commits at least one position, so L_total steps always suffice."""
