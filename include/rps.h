@@ -303,6 +303,25 @@ rps_status rps_decode_advance(const rps_pivots *piv, const rps_commit_out *commi
                               int32_t L_total, int32_t *d_tokens, int32_t *d_block, int32_t *d_mask_pos,
                               int32_t *d_mask_cnt, int32_t *d_done, int32_t *d_steps, rps_stream_t stream);
 
+/*
+ * Copy the rows of a row list from src to the same (req, branch, pos) of dst.
+ * The paper has no counterpart: it is data movement for callers whose logits
+ * sit in host memory, so that a step copies only the rows it scores (the masked
+ * base rows, then the lookahead rows rps_select_pivots lists) instead of the
+ * whole tensor, with no host synchronisation between the two. `rows` has the
+ * meaning of rps_score_step (mask form or explicit list; device arrays).
+ * src: device memory, or page-locked host memory (e.g. cudaHostAlloc), which the
+ * GPU reads through its device alias over the host link. dst: device memory
+ * (written, though rps_logits holds a const pointer).
+ * Same dtype, vocab and extents; strides may differ (16-byte multiples, 16-byte
+ * aligned bases).
+ * Errors: RPS_ERR_INVALID_ARG for NULL pointers, mismatched tensors, misaligned
+ * tensors, or src in pageable host memory (which the device cannot read
+ * safely); a row descriptor outside the tensors sets RPS_DEVERR_ROW_INDEX.
+ */
+rps_status rps_gather_rows(const rps_logits *src, const rps_row_list *rows, const rps_logits *dst,
+                           rps_stream_t stream);
+
 /* Bytes of scratch the library holds on each device for rps_score_step_noalloc. */
 #define RPS_STATIC_SCRATCH_BYTES (8u << 20)
 

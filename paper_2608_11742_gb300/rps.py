@@ -102,6 +102,8 @@ _lib.rps_score_and_commit.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.POINTER
 _lib.rps_decode_advance.restype = C.c_int
 _lib.rps_decode_advance.argtypes = [C.POINTER(RpsPivots), C.POINTER(RpsCommitOut), C.c_int32, C.c_int32, C.c_int32,
                                     _p, _p, _p, _p, _p, _p, _p]
+_lib.rps_gather_rows.restype = C.c_int
+_lib.rps_gather_rows.argtypes = [C.POINTER(RpsLogits), C.POINTER(RpsRowList), C.POINTER(RpsLogits), _p]
 _lib.rps_poll_device_status.restype = C.c_int
 _lib.rps_poll_device_status.argtypes = [_p, C.POINTER(C.c_uint32)]
 _lib.rps_status_string.restype = C.c_char_p
@@ -293,6 +295,20 @@ def rps_score_step_noalloc(logits: torch.Tensor, rows: Optional[torch.Tensor], s
            "rps_score_step_noalloc")
 
 
+def rps_gather_rows(src: torch.Tensor, rows: Optional[torch.Tensor], seg_cnt: Optional[torch.Tensor], n_seg: int,
+                    cap: int, dst: torch.Tensor, stream=None, mask_pos: Optional[torch.Tensor] = None,
+                    mask_branch: int = 0) -> None:
+    """Copy the listed rows of ``src`` (a CUDA tensor, or a page-locked CPU tensor the
+    GPU reads over the host link) into the same places of the CUDA tensor ``dst``."""
+    if src.shape != dst.shape or src.dtype != dst.dtype:
+        raise ValueError("src and dst must have the same shape and dtype")
+    if not src.is_cuda and not src.is_pinned():
+        raise ValueError("a host src must be page-locked (pin_memory)")
+    s, d = logits_desc(src), logits_desc(dst)
+    rl = RpsRowList(_ptr(rows), _ptr(seg_cnt), n_seg, cap, _ptr(mask_pos), mask_branch)
+    _check(_lib.rps_gather_rows(C.byref(s), C.byref(rl), C.byref(d), _stream(stream)), "rps_gather_rows")
+
+
 def rps_select_pivots(base: RowStatsBuf, n_req: int, L: int, mask_pos: torch.Tensor, mask_cnt: torch.Tensor, prm,
                       out: PivotsBuf, stream=None) -> None:
     b, p, o = base.c(), params(prm), out.c()
@@ -392,3 +408,17 @@ class Step:
         self.select(mask_pos, mask_cnt, stream)
         self.score_branch_rows(logits, stream)
         self.score_and_decide(logits, stream)
+
+    def run_host(self, host_logits, dev_logits, mask_pos, mask_cnt, stream=None):
+        """``run`` on logits that sit in page-locked host memory: only the rows the
+        step reads (the masked base rows, then the listed lookahead rows) are
+        gathered into ``dev_logits`` before they are scored; the lookahead list
+        stays on the device, so there is no host synchronisation in the step."""
+        n_req, L = self.n_req, self.L
+        rps_gather_rows(host_logits, None, mask_cnt, n_req, L, dev_logits, stream, mask_pos=mask_pos, mask_branch=0)
+        self.score_base(dev_logits, mask_pos, mask_cnt, stream)
+        self.select(mask_pos, mask_cnt, stream)
+        rps_gather_rows(host_logits, self.piv.branch_rows, self.piv.n_branch_rows, n_req, self.NB * L, dev_logits,
+                        stream)
+        self.score_branch_rows(dev_logits, stream)
+        self.score_and_decide(dev_logits, stream)
