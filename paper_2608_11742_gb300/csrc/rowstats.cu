@@ -118,6 +118,15 @@ __device__ __forceinline__ uint4 lds_again(const uint4 *p) {
     return v;
 }
 
+// 16-byte asynchronous global -> shared copy (L2 only), and the wait for all of
+// this thread's outstanding ones.
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
 }
@@ -254,6 +263,7 @@ struct LaneState {
     bool bad;         // NaN input seen (SAFE scan only)
     float c1v, c2v;   // top-k mode: this lane's two largest chunk maxima ...
     int c1u, c2u;     // ... and the first units of those chunks (-1 if none)
+    float c3v;        // top-k mode: its third largest chunk maximum (bounds every other chunk)
 };
 
 __device__ __forceinline__ void lane_init(LaneState &L) {
@@ -264,7 +274,7 @@ __device__ __forceinline__ void lane_init(LaneState &L) {
     L.best = -1;
     L.best_chunk = false;
     L.bad = false;
-    L.c1v = L.c2v = -INFINITY;
+    L.c1v = L.c2v = L.c3v = -INFINITY;
     L.c1u = L.c2u = -1;
 }
 
@@ -348,7 +358,10 @@ __device__ __forceinline__ float fold_chunk(LaneState &L, typename Elem<DT>::Ske
     raise_reference(L, cmax);
     if (TOPK && j0_valid(n_units, lane)) {
         sketch[cu + lane] = E::to_sketch(cmax);
-        if (cmax > L.c2v) {  // keep the two largest chunk maxima
+        if (cmax > L.c3v) {  // keep the three largest chunk maxima (first units of the top two)
+            L.c3v = fmaxf(L.c3v, fminf(cmax, L.c2v));
+        }
+        if (cmax > L.c2v) {
             if (cmax > L.c1v) {
                 L.c2v = L.c1v;
                 L.c2u = L.c1u;
@@ -393,13 +406,14 @@ __device__ void rescan_safe(LaneState &L, const char *row, int V, int u0, int u1
     constexpr int N = E::N;
     // the top-k chunk record of the fast pass stays valid: -inf and NaN do not
     // change a chunk's maximum
-    const float c1v = L.c1v, c2v = L.c2v;
+    const float c1v = L.c1v, c2v = L.c2v, c3v = L.c3v;
     const int c1u = L.c1u, c2u = L.c2u;
     lane_init(L);
     L.c1v = c1v;
     L.c2v = c2v;
     L.c1u = c1u;
     L.c2u = c2u;
+    L.c3v = c3v;
     const int full_end = min(u1, V / N);
     for (int u = u0 + lane; u < full_end; u += 32) {
         float y[N];
@@ -459,12 +473,18 @@ __device__ __forceinline__ void pair_step(float &v, int &i, int stride, bool kee
     }
 }
 
-__device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, int ci, int k, int lane) {
+__device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, int ci, int k, int lane,
+                                                 bool empty = false) {
 #pragma unroll
     for (int size = 2; size <= 32; size <<= 1) {
 #pragma unroll
         for (int stride = size >> 1; stride > 0; stride >>= 1)
             pair_step(cv, ci, stride, ((lane & size) == 0) == ((lane & stride) == 0));
+    }
+    if (empty) {  // the list held nothing: the sorted candidates are the list
+        tv = lane < k ? cv : -INFINITY;
+        ti = lane < k ? ci : INT_MAX;
+        return;
     }
     const float rv = __shfl_sync(kFull, cv, 31 - lane);
     const int ri = __shfl_sync(kFull, ci, 31 - lane);
@@ -482,27 +502,22 @@ __device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, i
 
 // Second pass of a segment (top-k mode). theta is a lower bound on the segment's
 // k-th largest logit, so only the (chunk, lane) pairs whose recorded maximum
-// reaches it can hold a member of the top k. Each lane loads kGroup of its
-// recorded maxima at once and marks its hits; then, round after round, every lane
-// with a hit left reloads that chunk's units (from L2) at the same time, and the
-// warp merges their elements at or above max(theta, current k-th entry) into the
-// warp-distributed list, 32 at a time (warp_merge_batch).
+// reaches it can hold a member of the top k.
+//
+// Bits j * N + i of the mask: element i of this lane's unit j of chunk cu
+// (staged at buf[j * 32 + lane]) is at or above th. Units are tested whole
+// first; most hold no such element.
 template <int DT>
-__device__ __forceinline__ void topk_round(const char *row, int cend, int cu, int k, int lane, float theta, float &tv,
-                                           int &ti, uint4 *stage, float2 *cand) {
+__device__ __forceinline__ unsigned long long cell_mask(const uint4 *buf, int cend, int cu, int lane, float th) {
     using E = Elem<DT>;
     constexpr int N = E::N;
-    static_assert(kBatch * N <= 64, "candidate mask holds 64 elements");
-    const uint32_t *words = reinterpret_cast<const uint32_t *>(stage);
-    const float th = fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
     unsigned long long cm = 0;
-    if (cu >= 0) {
+    if (cu < 0) return 0;
 #pragma unroll
-        for (int j = 0; j < kBatch; ++j) {
-            const int u = cu + j * 32 + lane;
-            if (u < cend) {
-                const uint4 w = ld_stream(row + static_cast<size_t>(u) * 16);
-                stage[lane * kBatch + j] = w;
+    for (int j = 0; j < kBatch; ++j) {
+        if (cu + j * 32 + lane < cend) {
+            const uint4 w = buf[j * 32 + lane];
+            if (E::unit_max(w) >= th) {
                 float y[N];
                 E::unpack(w, y);
 #pragma unroll
@@ -511,7 +526,24 @@ __device__ __forceinline__ void topk_round(const char *row, int cend, int cu, in
             }
         }
     }
-    // compact the round's candidates into the candidate buffer, then merge
+    return cm;
+}
+
+// Merges the elements at or above max(theta, current k-th entry) of up to two
+// staged chunks per lane (cu < 0: none) into the warp-distributed sorted list
+// (lane j = rank j), 32 at a time: the lanes compact their elements into the
+// candidate buffer, then warp_merge_batch. empty: the list holds nothing yet.
+template <int DT>
+__device__ __forceinline__ void topk_merge_cells(const uint4 *buf_a, int cu_a, const uint4 *buf_b, int cu_b, int cend,
+                                                 int k, int lane, float theta, float &tv, int &ti, float2 *cand,
+                                                 bool empty) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    constexpr int kCell = kBatch * N;
+    static_assert(2 * kCell <= 64, "candidate mask holds two chunks");
+    const float th = empty ? theta : fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
+    const unsigned long long cm =
+        cell_mask<DT>(buf_a, cend, cu_a, lane, th) | (cell_mask<DT>(buf_b, cend, cu_b, lane, th) << kCell);
     const int c = __popc(static_cast<unsigned>(cm)) + __popc(static_cast<unsigned>(cm >> 32));
     int incl = c;
 #pragma unroll
@@ -529,8 +561,12 @@ __device__ __forceinline__ void topk_round(const char *row, int cend, int cu, in
             const int bit = __ffsll(static_cast<long long>(bits)) - 1;
             bits &= bits - 1;
             if (slot >= done && slot < done + kCandBatch) {
-                const int j = bit / N, i = bit % N;
-                cand[slot - done] = make_float2(E::pick(words + (lane * kBatch + j) * 4, i),
+                const bool second = bit >= kCell;
+                const int e = second ? bit - kCell : bit;
+                const int j = e / N, i = e % N;
+                const uint32_t *words = reinterpret_cast<const uint32_t *>(second ? buf_b : buf_a);
+                const int cu = second ? cu_b : cu_a;
+                cand[slot - done] = make_float2(E::pick(words + (j * 32 + lane) * 4, i),
                                                 __int_as_float((cu + j * 32 + lane) * N + i));
             }
             ++slot;
@@ -538,26 +574,61 @@ __device__ __forceinline__ void topk_round(const char *row, int cend, int cu, in
         __syncwarp();
         const int idx = done + lane;
         const float2 e = idx < total ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
-        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane);
+        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane, empty && done == 0);
         __syncwarp();
     }
 }
 
+// Stage this lane's units of chunk cu in buf by asynchronous 16-byte copies
+// (cu < 0: none); complete with cp_async_wait_all.
+__device__ __forceinline__ void stage_async(uint4 *buf, const char *row, int cend, int cu, int lane) {
+    if (cu < 0) return;
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+        const int u = cu + j * 32 + lane;
+        if (u < cend) cp_async16(buf + j * 32 + lane, row + static_cast<size_t>(u) * 16);
+    }
+}
+
+// A reload round: stage chunk cu (per lane) in stage, then merge.
+template <int DT>
+__device__ __forceinline__ void topk_round(const char *row, int cend, int cu, int k, int lane, float theta, float &tv,
+                                           int &ti, uint4 *stage, float2 *cand) {
+    __syncwarp();
+    stage_async(stage, row, cend, cu, lane);
+    cp_async_wait_all();
+    topk_merge_cells<DT>(stage, cu, stage, -1, cend, k, lane, theta, tv, ti, cand, false);
+}
+
+// ring2: two idle ring buffers (the warp's piece is fully streamed) or null.
 template <int DT>
 __device__ void topk_from_sketch(const LaneState &L, const char *row, const typename Elem<DT>::Sketch *sketch, int u0,
                                  int cend, int k, int lane, float theta, float &tv, int &ti, uint4 *stage,
-                                 float2 *cand) {
+                                 float2 *cand, uint4 *ring2) {
     using E = Elem<DT>;
     constexpr int kGroup = 16;  // recorded maxima a lane loads together
     tv = -INFINITY;
     ti = INT_MAX;
     // Usually a lane's only chunks at or above the bound are its two best.
-    topk_round<DT>(row, cend, L.c1v >= theta ? L.c1u : -1, k, lane, theta, tv, ti, stage, cand);
-    if (__any_sync(kFull, L.c2v >= theta))
-        topk_round<DT>(row, cend, L.c2v >= theta ? L.c2u : -1, k, lane, theta, tv, ti, stage, cand);
-    // A lane whose second best chunk reaches the bound may have more: scan its
-    // recorded maxima for the rest.
-    const bool more = L.c2v >= theta;
+    const int cu1 = L.c1v >= theta ? L.c1u : -1;
+    const int cu2 = L.c2v >= theta ? L.c2u : -1;
+    if (ring2) {
+        // both reloads in flight at once
+        __syncwarp();
+        stage_async(ring2, row, cend, cu1, lane);
+        stage_async(ring2 + kChunkUnits, row, cend, cu2, lane);
+        cp_async_wait_all();
+        topk_merge_cells<DT>(ring2, cu1, ring2 + kChunkUnits, cu2, cend, k, lane, theta, tv, ti, cand, true);
+    } else {
+        __syncwarp();
+        stage_async(stage, row, cend, cu1, lane);
+        cp_async_wait_all();
+        topk_merge_cells<DT>(stage, cu1, stage, -1, cend, k, lane, theta, tv, ti, cand, true);
+        if (__any_sync(kFull, cu2 >= 0)) topk_round<DT>(row, cend, cu2, k, lane, theta, tv, ti, stage, cand);
+    }
+    // Every other chunk of a lane peaks at most at its third largest chunk
+    // maximum: scan the recorded maxima only where that reaches the bound.
+    const bool more = L.c3v >= fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
     if (!__any_sync(kFull, more)) return;
     for (int c0 = u0; c0 < cend; c0 += kGroup * kChunkUnits) {
         float m[kGroup];
@@ -693,15 +764,29 @@ __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, c
     }
 }
 
-// Merge of the top-k lists of every piece of a row (last arriver only), 32
-// entries per batch.
-__device__ __forceinline__ void merge_topk(const float2 *lists, int count, int k, int lane, float &tv, int &ti) {
-    const float2 e = __ldcg(lists + lane % k);  // list 0 seeds the merged list
-    tv = lane < k ? e.x : -INFINITY;
-    ti = lane < k ? __float_as_int(e.y) : INT_MAX;
+// Merge of the top-k lists of every piece of a row (last arriver only). The
+// k-th largest list head bounds the row's k-th largest logit from below (k
+// lists each hold an element at least that large), so only the entries that
+// reach it are compacted into the candidate buffer and merged, 32 at a time.
+__device__ __forceinline__ void merge_topk(const float2 *lists, int count, int k, int lane, float &tv, int &ti,
+                                           float2 *cand) {
     const int total = count * k;
-    constexpr int kPer = 4;  // batches whose entries are loaded together
-    for (int base = k; base < total; base += 32 * kPer) {
+    const float head = lane < count ? __ldcg(&lists[lane * k].x) : -INFINITY;
+    const float bound = count >= k ? warp_kth_largest(head, k, lane) : -INFINITY;
+    tv = -INFINITY;
+    ti = INT_MAX;
+    int filled = 0;
+    bool empty = true;
+    auto flush = [&]() {
+        __syncwarp();
+        const float2 e = lane < filled ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
+        __syncwarp();
+        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane, empty);
+        empty = false;
+        filled = 0;
+    };
+    constexpr int kPer = 4;  // entries a lane loads together
+    for (int base = 0; base < total; base += 32 * kPer) {
         float2 f[kPer];
 #pragma unroll
         for (int q = 0; q < kPer; ++q) {
@@ -709,9 +794,17 @@ __device__ __forceinline__ void merge_topk(const float2 *lists, int count, int k
             f[q] = idx < total ? __ldcg(lists + idx) : make_float2(-INFINITY, __int_as_float(INT_MAX));
         }
 #pragma unroll
-        for (int q = 0; q < kPer; ++q)
-            if (base + q * 32 < total) warp_merge_batch(tv, ti, f[q].x, __float_as_int(f[q].y), k, lane);
+        for (int q = 0; q < kPer; ++q) {
+            const bool keep = base + q * 32 + lane < total && f[q].x >= bound;
+            const unsigned b = __ballot_sync(kFull, keep);
+            const int n = __popc(b);
+            if (n == 0) continue;
+            if (filled + n > 32) flush();
+            if (keep) cand[filled + __popc(b & ((1u << lane) - 1u))] = f[q];
+            filled += n;
+        }
     }
+    if (filled > 0) flush();
 }
 
 // ---------------------------------------------------------------- segments
@@ -806,13 +899,13 @@ struct Producer {
 };
 
 template <int DT, bool TOPK>
-__global__ void __launch_bounds__(kRowThreads, 4) row_stats_kernel(const RowStatsArgs a) {
+__global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_stats_kernel(const RowStatsArgs a) {
     using E = Elem<DT>;
     constexpr int N = E::N;
     extern __shared__ __align__(128) uint4 dyn[];
     __shared__ int32_t seg_start[RPS_MAX_SEGMENTS + 1];
     __shared__ int32_t warp_total[kWarps];
-    constexpr int kRing = kStages;
+    constexpr int kRing = TOPK ? kStagesTopk : kStages;
     __shared__ __align__(8) uint64_t bars[kWarps][kRing];
 
     pdl_wait();
@@ -962,8 +1055,9 @@ __global__ void __launch_bounds__(kRowThreads, 4) row_stats_kernel(const RowStat
         int am;
         if (TOPK) {
             // the k-th largest lane maximum bounds the segment's k-th largest logit from below
+            // with nothing more in flight (the piece ends here) the ring stages the reloads
             topk_from_sketch<DT>(L, s.row, sketch, s.u0, cend, a.k, lane, warp_kth_largest(L.mx, a.k, lane), tv, ti,
-                                 stage, cand);
+                                 stage, cand, issued == acquired && kRing >= 2 ? ring : nullptr);
             if (s.u1 > full_units) topk_tail<DT>(s.row, V, a.k, lane, tv, ti);
             // rank 0 of T (largest logit, lowest token) is the argmax
             const float t0 = __shfl_sync(kFull, tv, 0);
@@ -1025,14 +1119,14 @@ __global__ void __launch_bounds__(kRowThreads, 4) row_stats_kernel(const RowStat
             p.amax = __ldcg(&part[lane].amax);
         }
         rt = combine(p.mref, p.s, p.t, p.mx, p.amax);
-        if (TOPK) merge_topk(a.part_topk + slot * kMaxPartials * a.k, count, a.k, lane, tv, ti);
+        if (TOPK) merge_topk(a.part_topk + slot * kMaxPartials * a.k, count, a.k, lane, tv, ti, cand);
         write_row(a, slot, rt, tv, ti, lane);
     }
 }
 
 template <int DT, bool TOPK>
 constexpr int dyn_smem_bytes() {
-    return kWarps * (kStages * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0)) *
+    return kWarps * ((TOPK ? kStagesTopk : kStages) * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0)) *
            static_cast<int>(sizeof(uint4));
 }
 

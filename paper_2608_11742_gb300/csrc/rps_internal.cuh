@@ -22,6 +22,14 @@ constexpr int kRowThreads = 256;   // threads per block of the row-statistics ke
 #endif
 constexpr int kBatch = RPS_RING_UNITS_PER_LANE;  // 16-byte units a lane takes from each ring buffer
 constexpr int kStages = RPS_RING_STAGES;         // ring buffers (bulk copies in flight) per warp
+#ifndef RPS_RING_STAGES_TOPK
+#define RPS_RING_STAGES_TOPK RPS_RING_STAGES
+#endif
+#ifndef RPS_TOPK_BLOCKS_PER_SM
+#define RPS_TOPK_BLOCKS_PER_SM 4
+#endif
+constexpr int kStagesTopk = RPS_RING_STAGES_TOPK;     // ring buffers per warp in top-k mode
+constexpr int kTopkBlocksPerSm = RPS_TOPK_BLOCKS_PER_SM;  // resident blocks the top-k kernel is compiled for
 
 // Partial statistics of one row segment, base-2 online softmax:
 // s = sum 2^u, t = sum u 2^u with u = (z - mref) * log2(e); mx = max z and
