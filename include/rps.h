@@ -16,6 +16,7 @@
  *                       with the eligible-commit count N_tau (Proposition 1)
  *   rps_commit          commit-or-abstain decision (Eq. 4 argmax over C
  *                       including [MASK]; Algorithm 1) and the mask after the step
+ *   rps_run_step        the whole step above in one call
  *
  * Conventions
  *   - Every array pointer is a caller-owned DEVICE pointer unless stated.
@@ -280,6 +281,24 @@ rps_status rps_score_and_commit(const rps_logits *anchor_logits, int32_t anchor_
                                 const rps_row_stats *anchor, const rps_row_stats *branch, int32_t n_req, int32_t L,
                                 const rps_pivots *piv, const rps_params *prm, const rps_branch_scores *scores,
                                 const rps_commit_out *out, rps_stream_t stream);
+
+/*
+ * One whole step in one call: rps_score_step over the base rows (branch 0 of
+ * `logits`, mask form d_mask_pos / d_mask_cnt of capacity L, top-k mode into
+ * `base`, workspace d_ws_base), rps_select_pivots into `piv`, rps_score_step
+ * over piv->branch_rows (statistics-only mode into `branch`, workspace
+ * d_ws_branch, a different one), and rps_score_and_commit with branch 0 as the
+ * anchor -- four launches with the results of the four calls. Every argument
+ * is checked before anything is enqueued. Because the call knows which launch
+ * writes what, the select launch stages the mask before waiting for the base
+ * statistics, and the score launch computes everything that does not read the
+ * lookahead statistics before waiting for them.
+ */
+rps_status rps_run_step(const rps_logits *logits, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
+                        const int32_t *d_mask_cnt, const rps_params *prm, const rps_row_stats *base,
+                        const rps_pivots *piv, const rps_row_stats *branch, const rps_branch_scores *scores,
+                        const rps_commit_out *out, void *d_ws_base, size_t ws_base_bytes, void *d_ws_branch,
+                        size_t ws_branch_bytes, rps_stream_t stream);
 
 /*
  * Outer loop of Algorithm 1 over semi-autoregressive blocks (the response of

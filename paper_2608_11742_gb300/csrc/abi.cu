@@ -127,8 +127,16 @@ rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream) 
     return from_cuda(cudaMemsetAsync(d_ws, 0, ws_bytes, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
-                          const rps_row_stats *out, void *d_ws, size_t ws_bytes, rps_stream_t stream) {
+}  // extern "C"
+
+namespace rps {
+namespace {
+
+// Checks the arguments of a row-statistics launch and fills its kernel
+// arguments and grid.
+rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                             const rps_row_stats *out, void *d_ws, size_t ws_bytes, RowStatsArgs *ap,
+                             int *grid_out) {
     rps_status st = check_logits(logits);
     if (st != RPS_OK) return st;
     if (!rows || (!rows->rows && !rows->mask_pos) || rows->n_seg < 1 || rows->cap < 1) return RPS_ERR_INVALID_ARG;
@@ -152,7 +160,7 @@ rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, co
     const int esize = logits->dtype == RPS_BF16 ? 2 : 4;
     const int per_unit = 16 / esize;
 
-    RowStatsArgs a;
+    RowStatsArgs &a = *ap;
     std::memset(&a, 0, sizeof a);
     a.data = logits->data;
     a.vocab = logits->vocab;
@@ -188,12 +196,33 @@ rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, co
     a.warps = grid * (kRowThreads / 32);
     a.min_piece = (a.units_per_row + (kMaxPartials - 2) - 1) / (kMaxPartials - 2);
     a.err = dev.err;
+    *grid_out = grid;
+    return RPS_OK;
+}
+
+}  // namespace
+}  // namespace rps
+
+extern "C" {
+
+rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                          const rps_row_stats *out, void *d_ws, size_t ws_bytes, rps_stream_t stream) {
+    RowStatsArgs a;
+    int grid = 0;
+    const rps_status st = prepare_row_stats(logits, rows, prm, out, d_ws, ws_bytes, &a, &grid);
+    if (st != RPS_OK) return st;
     return from_cuda(launch_row_stats(a, logits->dtype, grid, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
-                             const int32_t *d_mask_cnt, const rps_params *prm, const rps_pivots *out,
-                             rps_stream_t stream) {
+
+}  // extern "C"
+
+namespace rps {
+namespace {
+
+rps_status make_select_args(const rps_row_stats *base, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
+                            const int32_t *d_mask_cnt, const rps_params *prm, const rps_pivots *out,
+                            SelectArgs *ap) {
     rps_status st = check_params(prm, true);
     if (st != RPS_OK) return st;
     if (!base || !base->zmax || !base->pmax || !base->argmax || !base->mu || !base->htrunc || !base->H ||
@@ -207,7 +236,7 @@ rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L
         return RPS_ERR_INVALID_ARG;
     DeviceInfo dev;
     if ((st = device_info(&dev)) != RPS_OK) return st;
-    SelectArgs a;
+    SelectArgs &a = *ap;
     a.zmax = base->zmax;
     a.pmax = base->pmax;
     a.mu = base->mu;
@@ -231,8 +260,24 @@ rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L
     a.commit_k = prm->commit_k;
     a.out = *out;
     a.err = dev.err;
+    a.early = 0;
+    return RPS_OK;
+}
+
+}  // namespace
+}  // namespace rps
+
+extern "C" {
+
+rps_status rps_select_pivots(const rps_row_stats *base, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
+                             const int32_t *d_mask_cnt, const rps_params *prm, const rps_pivots *out,
+                             rps_stream_t stream) {
+    SelectArgs a;
+    const rps_status st = make_select_args(base, n_req, L, d_mask_pos, d_mask_cnt, prm, out, &a);
+    if (st != RPS_OK) return st;
     return from_cuda(launch_select(a, reinterpret_cast<cudaStream_t>(stream)));
 }
+
 
 }  // extern "C"
 
@@ -276,6 +321,7 @@ rps_status make_score_args(const rps_logits *anchor_logits, int32_t anchor_branc
     a->tau = prm->tau;
     a->out = *out;
     a->err = nullptr;
+    a->early = 0;
     return RPS_OK;
 }
 
@@ -343,6 +389,59 @@ rps_status rps_score_and_commit(const rps_logits *anchor_logits, int32_t anchor_
     if ((st = device_info(&dev)) != RPS_OK) return st;
     s.err = dev.err;
     return from_cuda(launch_score_commit(s, c, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+rps_status rps_run_step(const rps_logits *logits, int32_t n_req, int32_t L, const int32_t *d_mask_pos,
+                        const int32_t *d_mask_cnt, const rps_params *prm, const rps_row_stats *base,
+                        const rps_pivots *piv, const rps_row_stats *branch, const rps_branch_scores *scores,
+                        const rps_commit_out *out, void *d_ws_base, size_t ws_base_bytes, void *d_ws_branch,
+                        size_t ws_branch_bytes, rps_stream_t stream) {
+    // every argument is checked before anything is enqueued
+    if (!piv || !piv->branch_rows || !piv->n_branch_rows || !prm || !base || !base->topk_idx || !branch ||
+        branch->topk_idx)
+        return RPS_ERR_INVALID_ARG;
+    if (prm->n_pivots < 1 || prm->tokens_per_pivot < 1 || L < 1) return RPS_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(prm->n_pivots) * prm->tokens_per_pivot * L > INT32_MAX / 3) return RPS_ERR_INVALID_ARG;
+    rps_row_list rows_base;
+    rows_base.rows = nullptr;
+    rows_base.seg_cnt = d_mask_cnt;
+    rows_base.n_seg = n_req;
+    rows_base.cap = L;
+    rows_base.mask_pos = d_mask_pos;
+    rows_base.mask_branch = 0;
+    rps_row_list rows_la;
+    rows_la.rows = piv->branch_rows;
+    rows_la.seg_cnt = piv->n_branch_rows;
+    rows_la.n_seg = n_req;
+    rows_la.cap = prm->n_pivots * prm->tokens_per_pivot * L;
+    rows_la.mask_pos = nullptr;
+    rows_la.mask_branch = 0;
+    RowStatsArgs a_base, a_la;
+    SelectArgs sel;
+    ScoreArgs sc;
+    CommitArgs cm;
+    int grid_base = 0, grid_la = 0;
+    rps_status st;
+    if ((st = prepare_row_stats(logits, &rows_base, prm, base, d_ws_base, ws_base_bytes, &a_base, &grid_base)) != RPS_OK)
+        return st;
+    if ((st = make_select_args(base, n_req, L, d_mask_pos, d_mask_cnt, prm, piv, &sel)) != RPS_OK) return st;
+    if ((st = prepare_row_stats(logits, &rows_la, prm, branch, d_ws_branch, ws_branch_bytes, &a_la, &grid_la)) !=
+        RPS_OK)
+        return st;
+    if ((st = make_score_args(logits, 0, base, branch, n_req, L, piv, prm, scores, &sc)) != RPS_OK) return st;
+    if ((st = make_commit_args(scores, n_req, L, piv, prm, out, &cm)) != RPS_OK) return st;
+    if (d_ws_base == d_ws_branch) return RPS_ERR_INVALID_ARG;
+    sc.err = a_la.err;
+    // inside one step the select launch follows the base statistics only, and
+    // score and commit follow the lookahead statistics only
+    sel.early = 1;
+    sc.early = 1;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_row_stats(a_base, logits->dtype, grid_base, s);
+    if (e == cudaSuccess) e = launch_select(sel, s);
+    if (e == cudaSuccess) e = launch_row_stats(a_la, logits->dtype, grid_la, s);
+    if (e == cudaSuccess) e = launch_score_commit(sc, cm, s);
+    return from_cuda(e);
 }
 
 rps_status rps_poll_device_status(rps_stream_t stream, uint32_t *detail) {

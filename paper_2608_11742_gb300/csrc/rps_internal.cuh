@@ -84,6 +84,7 @@ struct SelectArgs {
     int32_t pivot_rule, commit_rule, commit_k;
     rps_pivots out;
     uint32_t *err;
+    int32_t early;  // the mask predates the previous launch (see select_kernel)
 };
 
 struct ScoreArgs {
@@ -98,6 +99,7 @@ struct ScoreArgs {
     float lambda, tau;
     rps_branch_scores out;
     uint32_t *err;
+    int32_t early;  // the pivots and anchor statistics predate the previous launch (see score_commit_kernel)
 };
 
 struct CommitArgs {

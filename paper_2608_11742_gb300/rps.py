@@ -99,6 +99,10 @@ _lib.rps_score_and_commit.restype = C.c_int
 _lib.rps_score_and_commit.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.POINTER(RpsRowStats),
                                       C.POINTER(RpsRowStats), C.c_int32, C.c_int32, C.POINTER(RpsPivots),
                                       C.POINTER(RpsParams), C.POINTER(RpsBranchScores), C.POINTER(RpsCommitOut), _p]
+_lib.rps_run_step.restype = C.c_int
+_lib.rps_run_step.argtypes = [C.POINTER(RpsLogits), C.c_int32, C.c_int32, _p, _p, C.POINTER(RpsParams),
+                              C.POINTER(RpsRowStats), C.POINTER(RpsPivots), C.POINTER(RpsRowStats),
+                              C.POINTER(RpsBranchScores), C.POINTER(RpsCommitOut), _p, C.c_size_t, _p, C.c_size_t, _p]
 _lib.rps_decode_advance.restype = C.c_int
 _lib.rps_decode_advance.argtypes = [C.POINTER(RpsPivots), C.POINTER(RpsCommitOut), C.c_int32, C.c_int32, C.c_int32,
                                     _p, _p, _p, _p, _p, _p, _p]
@@ -338,6 +342,17 @@ def rps_score_and_commit(anchor_logits: torch.Tensor, anchor_branch: int, anchor
                                      C.byref(p), C.byref(s), C.byref(o), _stream(stream)), "rps_score_and_commit")
 
 
+def rps_run_step(logits: torch.Tensor, n_req: int, L: int, mask_pos: torch.Tensor, mask_cnt: torch.Tensor, prm,
+                 base: RowStatsBuf, piv: PivotsBuf, branch: RowStatsBuf, scores: ScoresBuf, out: CommitBuf,
+                 ws_base: torch.Tensor, ws_branch: torch.Tensor, stream=None) -> None:
+    d, p = logits_desc(logits), params(prm)
+    b, pv, br, sc, o = base.c(), piv.c(), branch.c(), scores.c(), out.c()
+    _check(_lib.rps_run_step(C.byref(d), n_req, L, mask_pos.data_ptr(), mask_cnt.data_ptr(), C.byref(p), C.byref(b),
+                             C.byref(pv), C.byref(br), C.byref(sc), C.byref(o), ws_base.data_ptr(),
+                             ws_base.numel() * ws_base.element_size(), ws_branch.data_ptr(),
+                             ws_branch.numel() * ws_branch.element_size(), _stream(stream)), "rps_run_step")
+
+
 def rps_decode_advance(piv: PivotsBuf, commit: CommitBuf, n_req: int, B: int, L_total: int, tokens, block, mask_pos,
                        mask_cnt, done, steps=None, stream=None) -> None:
     pv, cm = piv.c(), commit.c()
@@ -356,12 +371,13 @@ def rps_poll_device_status(stream=None):
 
 # --------------------------------------------------------------------------- one step
 class Step:
-    """Preallocated buffers and the five ABI calls of one RPS decoding step.
+    """Preallocated buffers and the ABI calls of one RPS decoding step.
 
     The base branch (0) of ``logits`` is the anchor, as in the workloads here.
-    Kernels launched per ``run``: row statistics of the masked base rows (top-k
-    mode), pivot selection, row statistics of the lookahead rows, and branch
-    scores with the commit decision in one launch.
+    Kernels launched per ``run`` (one rps_run_step call): row statistics of the
+    masked base rows (top-k mode), pivot selection, row statistics of the
+    lookahead rows, and branch scores with the commit decision in one launch.
+    ``run_calls`` makes the same four launches through the separate calls.
     """
     LAUNCHES = 4
 
@@ -404,6 +420,10 @@ class Step:
                              self.commit, stream)
 
     def run(self, logits, mask_pos, mask_cnt, stream=None):
+        rps_run_step(logits, self.n_req, self.L, mask_pos, mask_cnt, self.prm, self.base, self.piv, self.branch,
+                     self.scores, self.commit, self.ws_base, self.ws_branch, stream)
+
+    def run_calls(self, logits, mask_pos, mask_cnt, stream=None):
         self.score_base(logits, mask_pos, mask_cnt, stream)
         self.select(mask_pos, mask_cnt, stream)
         self.score_branch_rows(logits, stream)

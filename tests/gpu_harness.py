@@ -188,6 +188,21 @@ def compare_commit(g: dict, o: dict, scores_o: dict, mask_L: int, what: str):
             assert near, f"{what}: commit of request {q} differs from the oracle away from any tie"
 
 
+def assert_same_step(a: rps.Step, b: rps.Step, what: str) -> None:
+    """Every output buffer of two steps is bit-identical (NaN matches NaN)."""
+    from dataclasses import fields
+    for part in ("base", "branch", "piv", "scores", "commit"):
+        x, y = getattr(a, part), getattr(b, part)
+        for f in fields(x):
+            tx, ty = getattr(x, f.name), getattr(y, f.name)
+            if tx is None:
+                assert ty is None
+                continue
+            same = torch.equal(tx.nan_to_num(-7.0), ty.nan_to_num(-7.0)) if tx.is_floating_point() else \
+                torch.equal(tx, ty)
+            assert same, f"{what}: {part}.{f.name} differs between rps_run_step and the separate calls"
+
+
 class GpuStep:
     """Runs one step through the C ABI and compares every stage with the oracle."""
 
@@ -221,6 +236,13 @@ class GpuStep:
             assert torch.equal(getattr(fused_sc, name).nan_to_num(-7.0), getattr(st.scores, name).nan_to_num(-7.0)), name
         for name in ("best_slot", "winner", "commit_pos", "commit_tok", "mask_cnt"):
             assert torch.equal(getattr(fused_cm, name), getattr(st.commit, name)), name
+        # rps_run_step (the same four kernels, two of them waiting later) gives
+        # exactly the results of the separate calls
+        one = rps.Step(self.n_req, self.L, self.V, prm, self.t.device, self.t.dtype)
+        one.run(self.t, self.d_mask_pos, self.d_mask_cnt)
+        status, detail = rps.rps_poll_device_status()
+        assert status == rps.RPS_OK, f"{what}: device error bits {detail:#x} (rps_run_step)"
+        assert_same_step(one, st, what)
 
         base_o = o.base_stats(self.logits_np, self.mask_pos, self.mask_cnt, prm.k_max)
         base_g = stats_np(st.base)
