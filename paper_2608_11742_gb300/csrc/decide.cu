@@ -11,12 +11,14 @@ namespace rps {
 namespace {
 
 // a.early: the mask predates the previous launch (the base rows' statistics),
-// so it is staged before waiting for that launch.
+// so it is staged before waiting for that launch. The next launch (the
+// lookahead rows' statistics) is released only at the end: its blocks would
+// otherwise sit, waiting, on this block's SM while it works.
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs a) {
     if (!a.early) pdl_wait();
-    pdl_launch_next();
     extern __shared__ __align__(16) unsigned char sel_smem[];
     select_request(a, blockIdx.x, sel_smem, a.early != 0);
+    pdl_launch_next();
 }
 
 __global__ void __launch_bounds__(kScoreThreads) score_kernel(const ScoreArgs a) {

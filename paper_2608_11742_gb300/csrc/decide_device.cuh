@@ -349,23 +349,33 @@ __device__ void select_request(const SelectArgs &a, int q, unsigned char *smem, 
     }
 
     // Step 6: branch b = j * K + c lists M' without pivot j; the lists of the
-    // valid branches are laid end to end in branch order.
-    if (tid == 0) {
+    // valid branches are laid end to end in branch order (one warp, 32
+    // branches at a time).
+    if (tid < 32) {
+        const int lane = tid;
         int off = 0, m = 0;
-        for (int b = 0; b < NB; ++b) {
+        for (int b0 = 0; b0 < NB; b0 += 32) {
+            const int b = b0 + lane;
             const int j = b / K, c = b % K;
-            const bool valid = j < n_piv && piv_nc[j] >= 2 && c < piv_nc[j];
-            const int n = valid ? n_rem - 1 : 0;
-            if (valid) valid_b[m++] = static_cast<int16_t>(b);
-            br_off[b] = off;
-            o.branch_off[q * NB + b] = off;
-            o.branch_cnt[q * NB + b] = n;
-            o.branch_valid[q * NB + b] = valid;
-            off += n;
+            const bool valid = b < NB && j < n_piv && piv_nc[j] >= 2 && c < piv_nc[j];
+            const unsigned vm = __ballot_sync(kFull, valid);
+            const int before = __popc(vm & ((1u << lane) - 1u));
+            if (b < NB) {
+                const int my_off = off + before * (n_rem - 1);
+                if (valid) valid_b[m + before] = static_cast<int16_t>(b);
+                br_off[b] = my_off;
+                o.branch_off[q * NB + b] = my_off;
+                o.branch_cnt[q * NB + b] = valid ? n_rem - 1 : 0;
+                o.branch_valid[q * NB + b] = valid;
+            }
+            off += __popc(vm) * (n_rem - 1);
+            m += __popc(vm);
         }
-        br_off[NB] = off;
-        o.n_branch_rows[q] = off;
-        o.state[q] = RPS_STATE_SEARCH;
+        if (lane == 0) {
+            br_off[NB] = off;
+            o.n_branch_rows[q] = off;
+            o.state[q] = RPS_STATE_SEARCH;
+        }
     }
     __syncthreads();
     // one warp per valid branch: M' in order, without the branch's pivot
