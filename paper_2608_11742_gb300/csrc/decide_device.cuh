@@ -81,6 +81,9 @@ __device__ Best block_best(Best mine, Best *buf) {
     return r;
 }
 
+// Brings the 128-byte line holding p into L1 (no data is returned).
+__device__ __forceinline__ void prefetch_l1(const void *p) { asm volatile("prefetch.global.L1 [%0];" ::"l"(p)); }
+
 // Pivot order as one unsigned key: larger truncated entropy first, then lower
 // position (positions are distinct). The float's bits are mapped to an unsigned
 // order; 0 is below every key and marks "none".
@@ -205,6 +208,13 @@ __device__ void select_request(const SelectArgs &a, int q, unsigned char *smem, 
         ht[k] = __ldcg(a.htrunc + base + k);
         hh[k] = __ldcg(a.H + base + k);
         am[k] = __ldcg(a.argmax + base + k);
+        // the pivots' candidate step reads a row's zmax and top-k list: bring
+        // them to L1 now, while the statistics load, instead of a round trip later
+        if (k < cnt) {
+            prefetch_l1(a.zmax + base + k);
+            prefetch_l1(a.topk_logit + (base + k) * a.k_max);
+            prefetch_l1(a.topk_idx + (base + k) * a.k_max);
+        }
     }
     __syncthreads();
 
@@ -322,12 +332,12 @@ __device__ void select_request(const SelectArgs &a, int q, unsigned char *smem, 
         const int lane = tid & 31, w = tid >> 5, nw = blockDim.x >> 5;
         for (int j = w; j < n_piv; j += nw) {
             const int64_t row = base + rk[piv_i[j]];
-            const double zmax = __ldcg(a.zmax + row);
+            const double zmax = a.zmax[row];
             bool pass = false;
             int tok = -1;
             if (lane < a.k_max) {
-                const double zt = __ldcg(a.topk_logit + row * a.k_max + lane);
-                tok = __ldcg(a.topk_idx + row * a.k_max + lane);
+                const double zt = a.topk_logit[row * a.k_max + lane];
+                tok = a.topk_idx[row * a.k_max + lane];
                 pass = zt - zmax >= a.log_r;
             }
             const unsigned m = __ballot_sync(kFull, pass);
