@@ -851,6 +851,27 @@ __device__ __forceinline__ void locate(const RowStatsArgs &a, const int32_t *seg
                     : nullptr;
 }
 
+// The cut of the rows' units into pieces, one per warp. Aligned: each row is
+// cut into equal pieces (at most ceil(nv / min_piece) per row), so that no
+// piece crosses a row boundary, where a warp's stream stops for the row's
+// record; taken when it leaves at most an eighth of the warps idle. Otherwise
+// all units are cut evenly (pieces of at least min_piece units). Returns the
+// units per piece.
+__device__ __forceinline__ int64_t piece_units(const RowStatsArgs &a, int64_t total_rows, int64_t nv,
+                                               bool &aligned) {
+    aligned = false;
+    if (total_rows <= a.warps) {
+        const int64_t ppr = min(static_cast<int64_t>(a.warps) / total_rows, (nv + a.min_piece - 1) / a.min_piece);
+        const int64_t piece = (nv + ppr - 1) / ppr;
+        const int64_t cpr = (nv + piece - 1) / piece;
+        if (8 * total_rows * cpr >= 7 * static_cast<int64_t>(a.warps)) {
+            aligned = true;
+            return piece;
+        }
+    }
+    return max((total_rows * nv + a.warps - 1) / a.warps, a.min_piece);
+}
+
 // Walks the row segments of the global unit range [g, g_end).
 template <int DT>
 __device__ __forceinline__ bool next_segment(const RowStatsArgs &a, const int32_t *seg_start, int64_t nv, int64_t &g,
@@ -961,10 +982,29 @@ __global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_
     const int64_t nv = a.units_per_row;
     const int64_t total = total_rows * nv;
     if (total == 0) return;
-    const int64_t piece = max((total + a.warps - 1) / a.warps, a.min_piece);
-    const int64_t g_begin = static_cast<int64_t>(warp) * piece;
-    if (g_begin >= total) return;
-    const int64_t g_end = min(g_begin + piece, total);
+    // With at least as many warps as rows, each row is cut into equal pieces
+    // (aligned: no piece crosses a row boundary, where a warp's stream would
+    // stop for the row's record); otherwise the units are cut evenly.
+    // (statistics-only mode: the top-k launch keeps the even cut, whose index
+    // arithmetic its registers are tuned for)
+    __shared__ int64_t cut_cpr[TOPK ? 1 : kWarps];  // pieces per row of an aligned cut, 0 for the even cut
+    if (!TOPK && lane == 0) cut_cpr[wib] = 0;
+    bool aligned = false;
+    const int64_t piece =
+        TOPK ? max((total + a.warps - 1) / a.warps, a.min_piece) : piece_units(a, total_rows, nv, aligned);
+    int64_t g_begin, g_end;
+    if (aligned) {
+        const int64_t cpr = (nv + piece - 1) / piece;  // pieces per row
+        const int64_t row0 = warp / cpr, part = warp % cpr;
+        if (row0 >= total_rows) return;
+        g_begin = row0 * nv + part * piece;
+        g_end = min(g_begin + piece, (row0 + 1) * nv);
+        if (lane == 0) cut_cpr[wib] = cpr;
+    } else {
+        g_begin = static_cast<int64_t>(warp) * piece;
+        if (g_begin >= total) return;
+        g_end = min(g_begin + piece, total);
+    }
     const int V = static_cast<int>(a.vocab);
     const int full_units = V / N;
 
@@ -1072,9 +1112,18 @@ __global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_
         unpack2(L.t, t_lo, t_hi);
         RowTotals rt = combine(L.mref, s_lo + s_hi, t_lo + t_hi, seg_mx, am);
 
-        const int64_t w_first = (r * nv) / piece;
-        const int64_t w_last = ((r + 1) * nv - 1) / piece;
-        const int count = static_cast<int>(w_last - w_first + 1);
+        // the pieces (warps) that hold a part of row r
+        int64_t w_first;
+        int count;
+        // (read back from shared memory so that it is not kept live through the stream)
+        const int64_t cpr = TOPK ? 0 : *reinterpret_cast<volatile int64_t *>(&cut_cpr[TOPK ? 0 : wib]);
+        if (cpr > 0) {
+            w_first = r * cpr;
+            count = static_cast<int>(cpr);
+        } else {
+            w_first = (r * nv) / piece;
+            count = static_cast<int>(((r + 1) * nv - 1) / piece - w_first + 1);
+        }
         const int64_t slot = s.slot;
         if (count == 1) {
             write_row(a, slot, rt, tv, ti, lane);
