@@ -193,7 +193,7 @@ rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows,
     a.sketch = k > 0 ? static_cast<void *>(ws + w.sketch) : nullptr;
     a.units_per_row = (logits->vocab + per_unit - 1) / per_unit;
     const int grid = dev.sm_count * dev.blocks[logits->dtype][topk ? 1 : 0];
-    a.warps = grid * (kRowThreads / 32);
+    a.warps = grid * (row_threads(topk) / 32);
     a.min_piece = (a.units_per_row + (kMaxPartials - 2) - 1) / (kMaxPartials - 2);
     a.err = dev.err;
     *grid_out = grid;

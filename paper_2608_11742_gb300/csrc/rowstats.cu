@@ -53,7 +53,6 @@ namespace {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kSlack = 8.0f;          // nats the reference may trail the maximum
-constexpr int kWarps = kRowThreads / 32;
 constexpr int kChunkUnits = 32 * kBatch;  // 16-byte units per ring buffer (2 KB)
 // Staging area of the top-k second pass (top-k mode only): a lane's units of one
 // chunk, then the round's candidates, kCandBatch (value, token) pairs at a time.
@@ -920,7 +919,9 @@ struct Producer {
 };
 
 template <int DT, bool TOPK>
-__global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_stats_kernel(const RowStatsArgs a) {
+__global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : kStatBlocksPerSm)
+    row_stats_kernel(const RowStatsArgs a) {
+    constexpr int kWarps = row_threads(TOPK) / 32;
     using E = Elem<DT>;
     constexpr int N = E::N;
     extern __shared__ __align__(128) uint4 dyn[];
@@ -943,7 +944,7 @@ __global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_
     // segments per thread, then a block-wide scan.
     int64_t total_rows;
     if (a.seg_cnt) {
-        constexpr int kPer = RPS_MAX_SEGMENTS / kRowThreads;
+        constexpr int kPer = RPS_MAX_SEGMENTS / row_threads(TOPK);
         int32_t c[kPer];
         int32_t local = 0;
 #pragma unroll
@@ -972,7 +973,7 @@ __global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_
             seg_start[threadIdx.x * kPer + i] = run;
             run += c[i];
         }
-        if (threadIdx.x == kRowThreads - 1) seg_start[RPS_MAX_SEGMENTS] = run;
+        if (threadIdx.x == row_threads(TOPK) - 1) seg_start[RPS_MAX_SEGMENTS] = run;
         __syncthreads();
         total_rows = seg_start[a.n_seg];
     } else {
@@ -1175,7 +1176,7 @@ __global__ void __launch_bounds__(kRowThreads, TOPK ? kTopkBlocksPerSm : 4) row_
 
 template <int DT, bool TOPK>
 constexpr int dyn_smem_bytes() {
-    return kWarps * ((TOPK ? kStagesTopk : kStages) * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0)) *
+    return row_threads(TOPK) / 32 * ((TOPK ? kStagesTopk : kStages) * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0)) *
            static_cast<int>(sizeof(uint4));
 }
 
@@ -1187,14 +1188,15 @@ cudaError_t prepare_typed() {
 
 template <int DT, bool TOPK>
 cudaError_t launch_typed(const RowStatsArgs &a, int grid, cudaStream_t stream) {
-    return launch_pdl(row_stats_kernel<DT, TOPK>, dim3(grid), dim3(kRowThreads), dyn_smem_bytes<DT, TOPK>(), stream, a);
+    return launch_pdl(row_stats_kernel<DT, TOPK>, dim3(grid), dim3(row_threads(TOPK)), dyn_smem_bytes<DT, TOPK>(), stream,
+                      a);
 }
 
 template <int DT, bool TOPK>
 cudaError_t occupancy_typed(int *blocks) {
     cudaError_t e = prepare_typed<DT, TOPK>();
     if (e != cudaSuccess) return e;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK>, kRowThreads,
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK>, row_threads(TOPK),
                                                          dyn_smem_bytes<DT, TOPK>());
 }
 

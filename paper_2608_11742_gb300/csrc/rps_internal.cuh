@@ -12,7 +12,16 @@ namespace rps {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kMaxPartials = 32;   // partial records per row (one merging warp)
-constexpr int kRowThreads = 256;   // threads per block of the row-statistics kernel
+constexpr int kRowThreads = 256;   // threads per block of the row-statistics kernel in top-k mode
+#ifndef RPS_STAT_THREADS
+#define RPS_STAT_THREADS 1024
+#endif
+constexpr int kStatThreads = RPS_STAT_THREADS;  // ... and in statistics-only mode (one block per SM: no launch-slot skew)
+#ifndef RPS_STAT_BLOCKS_PER_SM
+#define RPS_STAT_BLOCKS_PER_SM 1
+#endif
+constexpr int kStatBlocksPerSm = RPS_STAT_BLOCKS_PER_SM;
+__host__ __device__ constexpr int row_threads(bool topk) { return topk ? kRowThreads : kStatThreads; }
 // Shape of each warp's shared-memory ring (overridable at build time for tuning).
 #ifndef RPS_RING_UNITS_PER_LANE
 #define RPS_RING_UNITS_PER_LANE 4
