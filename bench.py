@@ -211,7 +211,7 @@ class Workload:
                  lambda: self.step.score_and_decide(self.logits))
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=self.stream):
-            self.step.run(self.logits, self.mpos, self.mcnt)  # the four launches of rps_run_step
+            self.step.run(self.logits, self.mpos, self.mcnt)  # the five launches of rps_run_step
         # the same step with an event node before and after every kernel
         self.graph_ev = torch.cuda.CUDAGraph()
         try:

@@ -1,6 +1,7 @@
 // abi.cu -- host side of the C ABI declared in include/rps.h: argument checks,
 // launch configuration, workspace layout and the device error word.
 #include <cmath>
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 
@@ -83,11 +84,12 @@ rps_status check_logits(const rps_logits *l) {
 }
 
 struct WorkspaceLayout {
-    size_t ticket, part, topk, sketch, total;
+    size_t ticket, part, topk, sketch, norm, piece, total;
 };
 
-// Tickets, partial records, per-piece top-k lists and the top-k sketch (one
-// element-sized entry per 16-byte unit of each row, of which a quarter is used).
+// Tickets, partial records, per-piece top-k lists, the top-k sketch (one
+// element-sized entry per cell: one lane's units of one 2 KB ring chunk) and
+// each row's softmax reference and sum.
 WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k) {
     WorkspaceLayout w;
     const size_t rows = static_cast<size_t>(max_rows);
@@ -97,7 +99,9 @@ WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k
     w.part = align_up(rows * sizeof(uint32_t));
     w.topk = w.part + align_up(rows * kMaxPartials * sizeof(Partial));
     w.sketch = w.topk + (k > 0 ? align_up(rows * kMaxPartials * static_cast<size_t>(k) * sizeof(float2)) : 0);
-    w.total = w.sketch + (k > 0 ? align_up(rows * units * esize) : 0);
+    w.norm = w.sketch + (k > 0 ? align_up(rows * static_cast<size_t>(sketch_entries(units)) * esize) : 0);
+    w.piece = w.norm + (k > 0 ? align_up(rows * sizeof(float4)) : 0);
+    w.total = w.piece + (k > 0 ? align_up(sizeof(int32_t)) : 0);
     return w;
 }
 
@@ -136,7 +140,7 @@ namespace {
 // arguments and grid.
 rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
                              const rps_row_stats *out, void *d_ws, size_t ws_bytes, RowStatsArgs *ap,
-                             int *grid_out) {
+                             int *grid_out, int *topk_grid_out) {
     rps_status st = check_logits(logits);
     if (st != RPS_OK) return st;
     if (!rows || (!rows->rows && !rows->mask_pos) || rows->n_seg < 1 || rows->cap < 1) return RPS_ERR_INVALID_ARG;
@@ -191,9 +195,16 @@ rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows,
     a.part = reinterpret_cast<Partial *>(ws + w.part);
     a.part_topk = k > 0 ? reinterpret_cast<float2 *>(ws + w.topk) : nullptr;
     a.sketch = k > 0 ? static_cast<void *>(ws + w.sketch) : nullptr;
+    a.norm = k > 0 ? reinterpret_cast<float4 *>(ws + w.norm) : nullptr;
+    a.sketch_piece = k > 0 ? reinterpret_cast<int32_t *>(ws + w.piece) : nullptr;
     a.units_per_row = (logits->vocab + per_unit - 1) / per_unit;
-    const int grid = dev.sm_count * dev.blocks[logits->dtype][topk ? 1 : 0];
-    a.warps = grid * (row_threads(topk) / 32);
+    a.sketch_stride = sketch_entries(a.units_per_row);
+    // split top-k mode streams the rows with the statistics-only launch
+    const bool fused = topk && !kTopkSplit;
+    const int grid = dev.sm_count * dev.blocks[logits->dtype][fused ? 1 : 0];
+    a.warps = grid * (row_threads(fused) / 32);
+    *topk_grid_out = static_cast<int>(std::min<int64_t>((max_rows + kTopkWarps - 1) / kTopkWarps,
+                                                         static_cast<int64_t>(dev.sm_count) * 16));
     a.min_piece = (a.units_per_row + (kMaxPartials - 2) - 1) / (kMaxPartials - 2);
     a.err = dev.err;
     *grid_out = grid;
@@ -208,10 +219,10 @@ extern "C" {
 rps_status rps_score_step(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
                           const rps_row_stats *out, void *d_ws, size_t ws_bytes, rps_stream_t stream) {
     RowStatsArgs a;
-    int grid = 0;
-    const rps_status st = prepare_row_stats(logits, rows, prm, out, d_ws, ws_bytes, &a, &grid);
+    int grid = 0, topk_grid = 0;
+    const rps_status st = prepare_row_stats(logits, rows, prm, out, d_ws, ws_bytes, &a, &grid, &topk_grid);
     if (st != RPS_OK) return st;
-    return from_cuda(launch_row_stats(a, logits->dtype, grid, reinterpret_cast<cudaStream_t>(stream)));
+    return from_cuda(launch_row_stats(a, logits->dtype, grid, topk_grid, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 
@@ -420,13 +431,14 @@ rps_status rps_run_step(const rps_logits *logits, int32_t n_req, int32_t L, cons
     SelectArgs sel;
     ScoreArgs sc;
     CommitArgs cm;
-    int grid_base = 0, grid_la = 0;
+    int grid_base = 0, grid_la = 0, topk_grid_base = 0, topk_grid_la = 0;
     rps_status st;
-    if ((st = prepare_row_stats(logits, &rows_base, prm, base, d_ws_base, ws_base_bytes, &a_base, &grid_base)) != RPS_OK)
+    if ((st = prepare_row_stats(logits, &rows_base, prm, base, d_ws_base, ws_base_bytes, &a_base, &grid_base,
+                                &topk_grid_base)) != RPS_OK)
         return st;
     if ((st = make_select_args(base, n_req, L, d_mask_pos, d_mask_cnt, prm, piv, &sel)) != RPS_OK) return st;
-    if ((st = prepare_row_stats(logits, &rows_la, prm, branch, d_ws_branch, ws_branch_bytes, &a_la, &grid_la)) !=
-        RPS_OK)
+    if ((st = prepare_row_stats(logits, &rows_la, prm, branch, d_ws_branch, ws_branch_bytes, &a_la, &grid_la,
+                                &topk_grid_la)) != RPS_OK)
         return st;
     if ((st = make_score_args(logits, 0, base, branch, n_req, L, piv, prm, scores, &sc)) != RPS_OK) return st;
     if ((st = make_commit_args(scores, n_req, L, piv, prm, out, &cm)) != RPS_OK) return st;
@@ -437,9 +449,9 @@ rps_status rps_run_step(const rps_logits *logits, int32_t n_req, int32_t L, cons
     sel.early = 1;
     sc.early = 1;
     const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    cudaError_t e = launch_row_stats(a_base, logits->dtype, grid_base, s);
+    cudaError_t e = launch_row_stats(a_base, logits->dtype, grid_base, topk_grid_base, s);
     if (e == cudaSuccess) e = launch_select(sel, s);
-    if (e == cudaSuccess) e = launch_row_stats(a_la, logits->dtype, grid_la, s);
+    if (e == cudaSuccess) e = launch_row_stats(a_la, logits->dtype, grid_la, topk_grid_la, s);
     if (e == cudaSuccess) e = launch_score_commit(sc, cm, s);
     return from_cuda(e);
 }

@@ -202,6 +202,7 @@ struct Elem<RPS_BF16> {
     }
     // per-(chunk, lane) maximum kept for the top-k second pass: the bf16 bits
     typedef uint16_t Sketch;
+    static constexpr uint32_t kNegInf2 = 0xff80ff80u;  // a 32-bit word of -inf sketch entries
     __device__ static __forceinline__ Sketch to_sketch(float v) { return static_cast<uint16_t>(__float_as_uint(v) >> 16); }
     __device__ static __forceinline__ float from_sketch(Sketch s) { return __uint_as_float(static_cast<uint32_t>(s) << 16); }
     // running maximum of whole units, kept as a packed bf16 pair
@@ -237,6 +238,7 @@ struct Elem<RPS_F32> {
         return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)), fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
     }
     typedef float Sketch;
+    static constexpr uint32_t kNegInf2 = 0xff800000u;
     __device__ static __forceinline__ Sketch to_sketch(float v) { return v; }
     __device__ static __forceinline__ float from_sketch(Sketch s) { return s; }
     typedef float Acc;
@@ -339,9 +341,10 @@ __device__ __forceinline__ void fold_unit(LaneState &L, const float (&y)[N], int
 
 // Fold this lane's units of one ring chunk (the fast path). The chunk's maximum
 // comes from packed compares; the exact argmax is resolved once per segment.
-template <int DT, bool TOPK>
+// SKETCH: every lane records its maximum (-inf without units) at key + lane.
+template <int DT, bool TOPK, bool SKETCH>
 __device__ __forceinline__ float fold_chunk(LaneState &L, typename Elem<DT>::Sketch *sketch, const uint4 *buf,
-                                            int n_units, int cu, int lane) {
+                                            int n_units, int cu, int key, int lane) {
     using E = Elem<DT>;
     constexpr int N = E::N;
     typename E::Acc acc = E::acc_init();
@@ -355,6 +358,7 @@ __device__ __forceinline__ float fold_chunk(LaneState &L, typename Elem<DT>::Ske
         L.best_chunk = true;
     }
     raise_reference(L, cmax);
+    if (SKETCH) sketch[key + lane] = E::to_sketch(cmax);
     if (TOPK && j0_valid(n_units, lane)) {
         sketch[cu + lane] = E::to_sketch(cmax);
         if (cmax > L.c3v) {  // keep the three largest chunk maxima (first units of the top two)
@@ -721,8 +725,25 @@ __device__ __forceinline__ RowTotals combine(float mref, float s, float t, float
     return r;
 }
 
+// mu (Eq. 3) and the truncated entropy of the warp's list (lane j = rank j)
+// against the row's reference B and sum S: p_v = 2^fma(z_v, log2(e), -B) / S.
+__device__ __forceinline__ void topk_mass(float tv, float M, float lnS, float invS, int k, int lane, float &mu,
+                                          float &ht) {
+    float p = 0.f, h = 0.f;
+    if (lane < k) {
+        const float u = fmaf(tv, kLog2e, -M);
+        p = ex2(u) * invS;
+        if (p > 0.f) h = -p * (u * kLn2 - lnS);
+    }
+    mu = warp_sum(p);
+    ht = warp_sum(h);
+}
+
+// SKETCH: the row's B, ln S, 1 / S and sketch segment 0 (len0) are kept for
+// the top-k launch.
+template <bool SKETCH = false>
 __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, const RowTotals &r, float tv, int ti,
-                                          int lane) {
+                                          int lane, int len0 = 0) {
     const bool ok = (r.MX > -INFINITY) && (r.S > 0.f) && !(r.S != r.S) && !(r.T != r.T) && (r.AM != INT_MAX);
     // Probabilities are formed against the reference B like the sums, p_v =
     // 2^fma(z_v, log2(e), -B) / S, never as exp(z_v - lse): with large logits
@@ -741,17 +762,13 @@ __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, c
         a.lse[slot] = lse;
         a.H[slot] = H;
         a.pmax[slot] = pmax;
-        a.argmax[slot] = ok ? r.AM : -1;
+        if (!SKETCH) a.argmax[slot] = ok ? r.AM : -1;
         if (!ok) flag_error(a.err, RPS_DEVERR_NONFINITE);
+        if (SKETCH) a.norm[slot] = make_float4(r.M, lnS, invS, __int_as_float(len0));
     }
-    if (a.k > 0) {
-        float p = 0.f, h = 0.f;
-        if (ok && lane < a.k) {
-            const float u = fmaf(tv, kLog2e, -r.M);
-            p = ex2(u) * invS;
-            if (p > 0.f) h = -p * (u * kLn2 - lnS);
-        }
-        const float mu = warp_sum(p), ht = warp_sum(h);
+    if (!SKETCH && a.k > 0) {
+        float mu, ht;
+        topk_mass(tv, r.M, lnS, invS, ok ? a.k : 0, lane, mu, ht);
         if (lane == 0) {
             a.mu[slot] = ok ? mu : NAN;
             a.htrunc[slot] = ok ? ht : NAN;
@@ -807,6 +824,48 @@ __device__ __forceinline__ void merge_topk(const float2 *lists, int count, int k
 }
 
 // ---------------------------------------------------------------- segments
+// Rows of the list: the exclusive prefix of the segment counts (clamped to
+// capacity) into seg_start, RPS_MAX_SEGMENTS / THREADS segments per thread and
+// a block-wide scan; returns the total. Every thread of the block must call it.
+template <int THREADS>
+__device__ __forceinline__ int64_t count_rows(const RowStatsArgs &a, int32_t *seg_start, int32_t *warp_total, int lane,
+                                              int wib) {
+    if (!a.seg_cnt) return static_cast<int64_t>(a.n_seg) * a.cap;
+    constexpr int kPer = RPS_MAX_SEGMENTS / THREADS;
+    static_assert(RPS_MAX_SEGMENTS % THREADS == 0, "segments split evenly over the threads");
+    int32_t c[kPer];
+    int32_t local = 0;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int sg = threadIdx.x * kPer + i;
+        int32_t v = sg < a.n_seg ? a.seg_cnt[sg] : 0;
+        if (v < 0 || v > a.cap) {
+            if (blockIdx.x == 0) flag_error(a.err, RPS_DEVERR_MASK);
+            v = v < 0 ? 0 : a.cap;
+        }
+        c[i] = v;
+        local += v;
+    }
+    int32_t incl = local;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t n = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += n;
+    }
+    if (lane == 31) warp_total[wib] = incl;
+    __syncthreads();
+    int32_t run = incl - local;
+    for (int w = 0; w < wib; ++w) run += warp_total[w];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        seg_start[threadIdx.x * kPer + i] = run;
+        run += c[i];
+    }
+    if (threadIdx.x == THREADS - 1) seg_start[RPS_MAX_SEGMENTS] = run;
+    __syncthreads();
+    return seg_start[a.n_seg];
+}
+
 struct Segment {
     int64_t slot;
     const char *row;
@@ -814,6 +873,29 @@ struct Segment {
     bool valid;   // false: skipped entry or bad descriptor
     bool bad;     // bad descriptor (to flag)
 };
+
+// The row of list entry s.slot of segment seg: validity and row pointer. CG:
+// loads through L2.
+template <int DT, bool CG = false>
+__device__ __forceinline__ void describe(const RowStatsArgs &a, int seg, Segment &s) {
+    int32_t req, br, pos;
+    if (a.rows) {
+        const int32_t *e = a.rows + s.slot * 3;
+        req = CG ? __ldcg(e) : e[0];
+        br = CG ? __ldcg(e + 1) : e[1];
+        pos = CG ? __ldcg(e + 2) : e[2];
+    } else {
+        req = seg;
+        br = a.mask_branch;
+        pos = CG ? __ldcg(a.mask_pos + s.slot) : a.mask_pos[s.slot];
+    }
+    s.bad = pos >= 0 && (req < 0 || req >= a.n_req || br < 0 || br >= a.n_branch || pos >= a.n_pos);
+    s.valid = pos >= 0 && !s.bad;
+    s.row = s.valid ? static_cast<const char *>(a.data) +
+                          (req * a.req_stride + br * a.branch_stride + static_cast<int64_t>(pos) * a.pos_stride) *
+                              Elem<DT>::kBytes
+                    : nullptr;
+}
 
 // Row r of the concatenated list -> (segment, entry) -> output slot and row pointer.
 template <int DT>
@@ -832,22 +914,7 @@ __device__ __forceinline__ void locate(const RowStatsArgs &a, const int32_t *seg
         seg = static_cast<int>(r / a.cap);
         s.slot = r;
     }
-    int32_t req, br, pos;
-    if (a.rows) {
-        req = a.rows[s.slot * 3 + 0];
-        br = a.rows[s.slot * 3 + 1];
-        pos = a.rows[s.slot * 3 + 2];
-    } else {
-        req = seg;
-        br = a.mask_branch;
-        pos = a.mask_pos[s.slot];
-    }
-    s.bad = pos >= 0 && (req < 0 || req >= a.n_req || br < 0 || br >= a.n_branch || pos >= a.n_pos);
-    s.valid = pos >= 0 && !s.bad;
-    s.row = s.valid ? static_cast<const char *>(a.data) +
-                          (req * a.req_stride + br * a.branch_stride + static_cast<int64_t>(pos) * a.pos_stride) *
-                              Elem<DT>::kBytes
-                    : nullptr;
+    describe<DT>(a, seg, s);
 }
 
 // The cut of the rows' units into pieces, one per warp. Aligned: each row is
@@ -869,6 +936,59 @@ __device__ __forceinline__ int64_t piece_units(const RowStatsArgs &a, int64_t to
         }
     }
     return max((total_rows * nv + a.warps - 1) / a.warps, a.min_piece);
+}
+
+// Sketch layout of one row under the cut of piece_units (top-k mode). The
+// pieces that hold a part of the row are its segments: segment 0 = [0, len0),
+// then pieces of `piece` units (the last one shorter). Each segment's ring
+// chunks start at the segment start; the sketch holds 32 entries per chunk,
+// segments in row order: ch0 chunks for segment 0, then cps per piece, then
+// -inf to the end of the slot's stride. The statistics launch passes len0 per
+// row and piece per launch to the top-k launch.
+struct SketchRow {
+    int len0;   // units of segment 0
+    int ch0;    // its chunks of whole units
+    int piece;  // units per further segment (the row length when there is none)
+    int cps;    // chunks per further segment
+};
+
+__device__ __forceinline__ SketchRow sketch_row(int len0, int piece, int full_units) {
+    SketchRow q;
+    q.len0 = len0;
+    q.ch0 = (min(len0, full_units) + kChunkUnits - 1) / kChunkUnits;
+    q.piece = piece;
+    q.cps = (piece + kChunkUnits - 1) / kChunkUnits;
+    return q;
+}
+
+// Segment 0 of row r under a cut of `piece` units per warp.
+__device__ __forceinline__ int sketch_len0(int64_t r, int64_t nv, int64_t piece, bool aligned) {
+    const int64_t off = aligned ? 0 : (r * nv) % piece;  // units of the first piece spent on earlier rows
+    return static_cast<int>(min(piece - off, nv));
+}
+
+// Sketch entry of the first chunk of the segment starting at unit u0.
+__device__ __forceinline__ int sketch_key(const SketchRow &q, int u0) {
+    return u0 == 0 ? 0 : 32 * (q.ch0 + (u0 - q.len0) / q.piece * q.cps);
+}
+
+// The units of sketch entry e of the row: first unit and count (units first +
+// 32 t, t < count, of one lane of one ring chunk).
+__device__ __forceinline__ void sketch_cell(const SketchRow &q, int full_units, int e, int &first, int &count) {
+    const int chunk = e >> 5, l = e & 31;
+    int cu, end;
+    if (chunk < q.ch0) {
+        cu = chunk * kChunkUnits;
+        end = q.len0;
+    } else {
+        const int j = (chunk - q.ch0) / q.cps;
+        const int s0 = q.len0 + j * q.piece;
+        cu = s0 + (chunk - q.ch0 - j * q.cps) * kChunkUnits;
+        end = s0 + q.piece;
+    }
+    end = min(min(end, cu + kChunkUnits), full_units);
+    first = cu + l;
+    count = first < end ? min((end - first + 31) / 32, kBatch) : 0;
 }
 
 // Walks the row segments of the global unit range [g, g_end).
@@ -918,7 +1038,9 @@ struct Producer {
     }
 };
 
-template <int DT, bool TOPK>
+// SKETCH (statistics-only, first launch of split top-k mode): also the sketch
+// (layout of sketch_row) and each row's B, ln S and 1 / S for the top-k launch.
+template <int DT, bool TOPK, bool SKETCH>
 __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : kStatBlocksPerSm)
     row_stats_kernel(const RowStatsArgs a) {
     constexpr int kWarps = row_threads(TOPK) / 32;
@@ -940,45 +1062,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
     float2 *cand = reinterpret_cast<float2 *>(stage + kStageUnits);
     uint64_t *bar = bars[wib];
 
-    // Exclusive prefix of the segment counts (clamped to capacity), four
-    // segments per thread, then a block-wide scan.
-    int64_t total_rows;
-    if (a.seg_cnt) {
-        constexpr int kPer = RPS_MAX_SEGMENTS / row_threads(TOPK);
-        int32_t c[kPer];
-        int32_t local = 0;
-#pragma unroll
-        for (int i = 0; i < kPer; ++i) {
-            const int s = threadIdx.x * kPer + i;
-            int32_t v = s < a.n_seg ? a.seg_cnt[s] : 0;
-            if (v < 0 || v > a.cap) {
-                if (blockIdx.x == 0) flag_error(a.err, RPS_DEVERR_MASK);
-                v = v < 0 ? 0 : a.cap;
-            }
-            c[i] = v;
-            local += v;
-        }
-        int32_t incl = local;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int32_t n = __shfl_up_sync(kFull, incl, o);
-            if (lane >= o) incl += n;
-        }
-        if (lane == 31) warp_total[wib] = incl;
-        __syncthreads();
-        int32_t run = incl - local;
-        for (int w = 0; w < wib; ++w) run += warp_total[w];
-#pragma unroll
-        for (int i = 0; i < kPer; ++i) {
-            seg_start[threadIdx.x * kPer + i] = run;
-            run += c[i];
-        }
-        if (threadIdx.x == row_threads(TOPK) - 1) seg_start[RPS_MAX_SEGMENTS] = run;
-        __syncthreads();
-        total_rows = seg_start[a.n_seg];
-    } else {
-        total_rows = static_cast<int64_t>(a.n_seg) * a.cap;
-    }
+    const int64_t total_rows = count_rows<row_threads(TOPK)>(a, seg_start, warp_total, lane, wib);
 
     const int64_t nv = a.units_per_row;
     const int64_t total = total_rows * nv;
@@ -993,6 +1077,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
     bool aligned = false;
     const int64_t piece =
         TOPK ? max((total + a.warps - 1) / a.warps, a.min_piece) : piece_units(a, total_rows, nv, aligned);
+    if (SKETCH && blockIdx.x == 0 && threadIdx.x == 0) *a.sketch_piece = static_cast<int>(min(piece, nv));
     int64_t g_begin, g_end;
     if (aligned) {
         const int64_t cpr = (nv + piece - 1) / piece;  // pieces per row
@@ -1071,13 +1156,26 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
         }
         LaneState L;
         lane_init(L);
-        typename E::Sketch *sketch = TOPK ? static_cast<typename E::Sketch *>(a.sketch) + s.slot * nv : nullptr;
+        typename E::Sketch *sketch =
+            TOPK || SKETCH ? static_cast<typename E::Sketch *>(a.sketch) + s.slot * a.sketch_stride : nullptr;
         const int cend = min(s.u1, full_units);
+        int key = SKETCH ? sketch_key(sketch_row(sketch_len0(r, nv, piece, aligned), static_cast<int>(min(piece, nv)),
+                                                 full_units),
+                                      s.u0)
+                         : 0;
         for (int cu = s.u0; cu < cend; cu += kChunkUnits) {
             int st;
             if (!acquire(st)) return;
-            fold_chunk<DT, TOPK>(L, sketch, ring + st * kChunkUnits, min(kChunkUnits, cend - cu), cu, lane);
+            fold_chunk<DT, TOPK, SKETCH>(L, sketch, ring + st * kChunkUnits, min(kChunkUnits, cend - cu), cu, key,
+                                         lane);
+            key += 32;
             release();
+        }
+        if (SKETCH && s.u1 == nv) {  // the rest of the slot's sketch reads as -inf
+            constexpr int kPerVec = 16 / static_cast<int>(sizeof(typename E::Sketch));
+            uint4 *p = reinterpret_cast<uint4 *>(sketch);
+            const uint4 ninf = make_uint4(E::kNegInf2, E::kNegInf2, E::kNegInf2, E::kNegInf2);
+            for (int v = key / kPerVec + lane; v < a.sketch_stride / kPerVec; v += 32) p[v] = ninf;
         }
         if (s.u1 > full_units) fold_tail<DT, false>(L, s.row, V, lane);
         {
@@ -1105,6 +1203,8 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
             const int i0 = __shfl_sync(kFull, ti, 0);
             seg_mx = lane == 0 ? t0 : -INFINITY;
             am = lane == 0 ? i0 : INT_MAX;
+        } else if (SKETCH) {
+            am = 0;  // the top-k launch takes the argmax from its list
         } else {
             am = resolve_argmax<DT>(s.row, V, L, warp_max(L.mx), lane);
         }
@@ -1127,7 +1227,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
         }
         const int64_t slot = s.slot;
         if (count == 1) {
-            write_row(a, slot, rt, tv, ti, lane);
+            write_row<SKETCH>(a, slot, rt, tv, ti, lane, SKETCH ? sketch_len0(r, nv, piece, aligned) : 0);
             continue;
         }
         const int my = static_cast<int>(warp - w_first);
@@ -1170,7 +1270,266 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
         }
         rt = combine(p.mref, p.s, p.t, p.mx, p.amax);
         if (TOPK) merge_topk(a.part_topk + slot * kMaxPartials * a.k, count, a.k, lane, tv, ti, cand);
-        write_row(a, slot, rt, tv, ti, lane);
+        write_row<SKETCH>(a, slot, rt, tv, ti, lane, SKETCH ? sketch_len0(r, nv, piece, aligned) : 0);
+    }
+}
+
+// ---------------------------------------------------------------- top-k launch
+// Second launch of top-k mode (k <= 32), one warp per row. Its statistics
+// launch left the row's sketch -- the maximum of every cell, a cell being one
+// lane's units of one ring chunk -- and B, ln S, 1 / S. The k-th largest of the 32
+// lanes' largest sketch entries bounds the row's k-th largest logit from below
+// (k lanes each saw a different cell holding an element at least that large),
+// so only the cells whose maximum reaches the bound -- about k of them -- are
+// read again, and their elements at or above it enter the warp-distributed
+// sorted list (lane j = rank j, logit desc then token asc).
+constexpr int kCellCap = 256;  // candidate cells a warp buffers before reloading them
+constexpr int kSketchVecs = 24;  // 16-byte sketch loads a lane keeps in flight (a slot of <= 768 in one go)
+static_assert(kSketchVecs <= 32, "one hit bit per vector");
+
+// Merges the elements at or above max(theta, current k-th entry) of the staged
+// cells (lane j: units first + 32 t at stage[t * 32 + j], t < count).
+template <int DT>
+__device__ __forceinline__ void merge_staged_cells(const uint4 *stage, int first, int count, int k, int lane,
+                                                   float theta, float &tv, int &ti, float2 *cand, bool &empty) {
+    using E = Elem<DT>;
+    constexpr int N = E::N;
+    static_assert(kBatch * N <= 32, "a cell's elements fit one mask word");
+    const float th = empty ? theta : fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
+    uint32_t cm = 0;
+#pragma unroll
+    for (int t = 0; t < kBatch; ++t) {
+        if (t < count) {
+            const uint4 w = stage[t * 32 + lane];
+            if (E::unit_max(w) >= th) {
+                float y[N];
+                E::unpack(w, y);
+#pragma unroll
+                for (int i = 0; i < N; ++i)
+                    if (y[i] >= th) cm |= 1u << (t * N + i);
+            }
+        }
+    }
+    const int c = __popc(cm);
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += n;
+    }
+    const int total = __shfl_sync(kFull, incl, 31);
+    const uint32_t *words = reinterpret_cast<const uint32_t *>(stage);
+    for (int done = 0; done < total; done += kCandBatch) {
+        int slot = incl - c;
+        uint32_t bits = cm;
+        while (bits) {
+            const int bit = __ffs(bits) - 1;
+            bits &= bits - 1;
+            if (slot >= done && slot < done + kCandBatch) {
+                const int t = bit / N, i = bit % N;
+                cand[slot - done] = make_float2(E::pick(words + (t * 32 + lane) * 4, i),
+                                                __int_as_float((first + 32 * t) * N + i));
+            }
+            ++slot;
+        }
+        __syncwarp();
+        const float2 e = done + lane < total ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
+        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane, empty);
+        empty = false;
+        __syncwarp();
+    }
+}
+
+// Reloads the buffered cells cells[0, n) (sketch entries), 32 at a time, and
+// merges their elements.
+template <int DT>
+__device__ void merge_sketch_cells(const char *row, const int32_t *cells, int n, const SketchRow &cut, int full_units,
+                                   int k, int lane, float theta, float &tv, int &ti, uint4 *stage, float2 *cand,
+                                   bool &empty) {
+    for (int b = 0; b < n; b += 32) {
+        int first = 0, count = 0;
+        if (b + lane < n) sketch_cell(cut, full_units, cells[b + lane], first, count);
+        __syncwarp();
+#pragma unroll
+        for (int t = 0; t < kBatch; ++t)
+            if (t < count) cp_async16(stage + t * 32 + lane, row + static_cast<size_t>(first + 32 * t) * 16);
+        cp_async_wait_all();
+        __syncwarp();
+        merge_staged_cells<DT>(stage, first, count, k, lane, theta, tv, ti, cand, empty);
+    }
+}
+
+// The largest entry of each of this lane's sketch vectors v0 + 32 q + lane
+// (-inf past the row's n_vec).
+template <int DT>
+__device__ __forceinline__ void vector_maxima(float (&vm)[kSketchVecs], const uint4 *sk, int v0, int n_vec, int lane) {
+    uint4 w[kSketchVecs];
+#pragma unroll
+    for (int q = 0; q < kSketchVecs; ++q) {
+        const int v = v0 + q * 32 + lane;
+        w[q] = v < n_vec ? __ldg(sk + v) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int q = 0; q < kSketchVecs; ++q) vm[q] = v0 + q * 32 + lane < n_vec ? Elem<DT>::unit_max(w[q]) : -INFINITY;
+}
+
+// Bit i: entry i of sketch vector *p reaches theta.
+template <int DT>
+__device__ __forceinline__ uint32_t vector_hits(const uint4 *p, float theta) {
+    constexpr int kPerVec = 16 / static_cast<int>(sizeof(typename Elem<DT>::Sketch));
+    float y[kPerVec];
+    Elem<DT>::unpack(__ldg(p), y);
+    uint32_t m = 0;
+#pragma unroll
+    for (int i = 0; i < kPerVec; ++i)
+        if (y[i] >= theta) m |= 1u << i;
+    return m;
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kTopkWarps * 32, kTopkMinBlocks) topk_rows_kernel(const RowStatsArgs a) {
+    using E = Elem<DT>;
+    constexpr int kPerVec = 16 / static_cast<int>(sizeof(typename E::Sketch));  // sketch entries per 16 bytes
+    __shared__ uint4 stage_all[kTopkWarps][kBatch * 32];
+    __shared__ float2 cand_all[kTopkWarps][kCandBatch];
+    __shared__ int32_t cells_all[kTopkWarps][kCellCap];
+
+    const int lane = threadIdx.x & 31;
+    const int wib = threadIdx.x >> 5;
+    uint4 *stage = stage_all[wib];
+    float2 *cand = cand_all[wib];
+    int32_t *cells = cells_all[wib];
+    const int64_t n_slots = static_cast<int64_t>(a.n_seg) * a.cap;
+    const int64_t nv = a.units_per_row;
+    const int V = static_cast<int>(a.vocab);
+    const int full_units = V / Elem<DT>::N;
+    const int k = a.k;
+    const int n_vec = static_cast<int>(a.sketch_stride / kPerVec);  // the whole slot (-inf past the row's chunks)
+    const bool one_batch = n_vec <= 32 * kSketchVecs;
+    bool waited = false;
+
+    // One warp per list slot (entry), in slot order: no scan of the list.
+    for (int64_t slot = static_cast<int64_t>(blockIdx.x) * kTopkWarps + wib;;
+         slot += static_cast<int64_t>(gridDim.x) * kTopkWarps) {
+        // The list is an input of the statistics launch, which waited for its
+        // producers before letting this launch begin: it is read before the wait.
+        Segment s;
+        s.slot = slot;
+        s.valid = false;
+        const bool have = slot < n_slots;
+        if (have) {
+            const int seg = static_cast<int>(slot / a.cap);
+            int cnt = a.cap;
+            if (a.seg_cnt) cnt = min(max(__ldcg(a.seg_cnt + seg), 0), a.cap);  // (as the statistics launch clamps)
+            if (slot - static_cast<int64_t>(seg) * a.cap < cnt) describe<DT, true>(a, seg, s);
+        }
+        if (!waited) {  // everything below reads the statistics launch's results
+            pdl_wait();
+            pdl_launch_next();
+            waited = true;
+        }
+        if (!have) break;
+        if (!s.valid) continue;  // skipped entry, or a bad descriptor the statistics launch flagged
+        const uint4 *sk = reinterpret_cast<const uint4 *>(static_cast<const typename E::Sketch *>(a.sketch) +
+                                                          slot * a.sketch_stride);
+        const float zmax = __ldcg(a.zmax + slot);
+        const float4 nrm = __ldcg(a.norm + slot);
+        const int piece = __ldcg(a.sketch_piece);
+        // Pass 1: the largest entry of each of this lane's vectors v0 + 32 q + lane.
+        float vm[kSketchVecs];
+        vector_maxima<DT>(vm, sk, 0, n_vec, lane);
+        if (zmax != zmax) {  // the statistics launch found no finite row
+            if (lane == 0) {
+                a.argmax[slot] = -1;
+                a.mu[slot] = NAN;
+                a.htrunc[slot] = NAN;
+            }
+            if (lane < k) {
+                a.topk_idx[slot * k + lane] = -1;
+                a.topk_logit[slot * k + lane] = NAN;
+            }
+            continue;
+        }
+        const SketchRow cut = sketch_row(__float_as_int(nrm.w), piece, full_units);
+        // the k-th largest of the lanes' largest entries
+        float lane_max = -INFINITY;
+        for (int v0 = 0;;) {
+#pragma unroll
+            for (int q = 0; q < kSketchVecs; ++q) lane_max = fmaxf(lane_max, vm[q]);
+            v0 += 32 * kSketchVecs;
+            if (v0 >= n_vec) break;
+            vector_maxima<DT>(vm, sk, v0, n_vec, lane);
+        }
+        const float theta = warp_kth_largest(lane_max, k, lane);
+
+        // Pass 2: the cells that reach it, buffered and reloaded kCellCap at a
+        // time. Few vectors hold one; only those are read again (from L1).
+        float tv = -INFINITY;
+        int ti = INT_MAX;
+        bool empty = true;
+        int pending = 0;
+        for (int v0 = 0; v0 < n_vec; v0 += 32 * kSketchVecs) {
+            if (!one_batch) vector_maxima<DT>(vm, sk, v0, n_vec, lane);
+            uint32_t hv = 0;  // bit q: vector q holds an entry at or above theta
+#pragma unroll
+            for (int q = 0; q < kSketchVecs; ++q)
+                if (vm[q] >= theta) hv |= 1u << q;
+            if (!__any_sync(kFull, hv != 0)) continue;
+            int c = 0;
+            for (uint32_t b = hv; b; b &= b - 1) c += __popc(vector_hits<DT>(sk + v0 + (__ffs(b) - 1) * 32 + lane, theta));
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int n = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += n;
+            }
+            const int end = pending + __shfl_sync(kFull, incl, 31);
+            for (int base = 0;; base += kCellCap) {
+                int slot_i = pending + incl - c;
+                for (uint32_t b = hv; b; b &= b - 1) {
+                    const int q = __ffs(b) - 1;
+                    uint32_t m = vector_hits<DT>(sk + v0 + q * 32 + lane, theta);
+                    while (m) {
+                        const int i = __ffs(m) - 1;
+                        m &= m - 1;
+                        if (slot_i >= base && slot_i < base + kCellCap)
+                            cells[slot_i - base] = (v0 + q * 32 + lane) * kPerVec + i;
+                        ++slot_i;
+                    }
+                }
+                __syncwarp();
+                if (end - base <= kCellCap) {
+                    pending = end - base;
+                    break;
+                }
+                merge_sketch_cells<DT>(s.row, cells, kCellCap, cut, full_units, k, lane, theta, tv, ti, stage, cand,
+                                       empty);
+                __syncwarp();
+            }
+            if (pending == kCellCap) {
+                merge_sketch_cells<DT>(s.row, cells, kCellCap, cut, full_units, k, lane, theta, tv, ti, stage, cand,
+                                       empty);
+                pending = 0;
+                __syncwarp();
+            }
+        }
+        if (pending > 0)
+            merge_sketch_cells<DT>(s.row, cells, pending, cut, full_units, k, lane, theta, tv, ti, stage, cand, empty);
+        if (full_units < nv) topk_tail<DT>(s.row, V, k, lane, tv, ti);
+
+        float mu, ht;
+        topk_mass(tv, nrm.x, nrm.y, nrm.z, k, lane, mu, ht);
+        // rank 0 of T (largest logit, lowest token) is the argmax of Eq. 1
+        const int i0 = __shfl_sync(kFull, ti, 0);
+        if (lane == 0) {
+            a.argmax[slot] = i0;
+            a.mu[slot] = mu;
+            a.htrunc[slot] = ht;
+        }
+        if (lane < k) {
+            a.topk_idx[slot * k + lane] = ti;
+            a.topk_logit[slot * k + lane] = tv;
+        }
     }
 }
 
@@ -1180,32 +1539,49 @@ constexpr int dyn_smem_bytes() {
            static_cast<int>(sizeof(uint4));
 }
 
-template <int DT, bool TOPK>
+template <int DT, bool TOPK, bool SKETCH = false>
 cudaError_t prepare_typed() {
-    return cudaFuncSetAttribute(row_stats_kernel<DT, TOPK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    return cudaFuncSetAttribute(row_stats_kernel<DT, TOPK, SKETCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 dyn_smem_bytes<DT, TOPK>());
 }
 
-template <int DT, bool TOPK>
+template <int DT, bool TOPK, bool SKETCH = false>
 cudaError_t launch_typed(const RowStatsArgs &a, int grid, cudaStream_t stream) {
-    return launch_pdl(row_stats_kernel<DT, TOPK>, dim3(grid), dim3(row_threads(TOPK)), dyn_smem_bytes<DT, TOPK>(), stream,
-                      a);
+    return launch_pdl(row_stats_kernel<DT, TOPK, SKETCH>, dim3(grid), dim3(row_threads(TOPK)),
+                      dyn_smem_bytes<DT, TOPK>(), stream, a);
+}
+
+// Top-k mode as two launches: statistics with the sketch, then the top-k rows.
+template <int DT>
+cudaError_t launch_split(const RowStatsArgs &a, int grid, int topk_grid, cudaStream_t stream) {
+    RowStatsArgs st = a;
+    st.k = 0;
+    cudaError_t e = launch_typed<DT, false, true>(st, grid, stream);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(topk_rows_kernel<DT>, dim3(topk_grid), dim3(kTopkWarps * 32), 0, stream, a);
 }
 
 template <int DT, bool TOPK>
 cudaError_t occupancy_typed(int *blocks) {
     cudaError_t e = prepare_typed<DT, TOPK>();
     if (e != cudaSuccess) return e;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK>, row_threads(TOPK),
+    if (!TOPK && (e = prepare_typed<DT, false, true>()) != cudaSuccess) return e;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK, false>, row_threads(TOPK),
                                                          dyn_smem_bytes<DT, TOPK>());
+}
+
+template <int DT>
+cudaError_t launch_dtype(const RowStatsArgs &a, int grid, int topk_grid, cudaStream_t stream) {
+    if (a.k == 0) return launch_typed<DT, false>(a, grid, stream);
+    if (kTopkSplit) return launch_split<DT>(a, grid, topk_grid, stream);
+    return launch_typed<DT, true>(a, grid, stream);
 }
 
 }  // namespace
 
-cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, cudaStream_t stream) {
-    if (dtype == RPS_BF16)
-        return a.k > 0 ? launch_typed<RPS_BF16, true>(a, grid, stream) : launch_typed<RPS_BF16, false>(a, grid, stream);
-    return a.k > 0 ? launch_typed<RPS_F32, true>(a, grid, stream) : launch_typed<RPS_F32, false>(a, grid, stream);
+cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, int topk_grid, cudaStream_t stream) {
+    return dtype == RPS_BF16 ? launch_dtype<RPS_BF16>(a, grid, topk_grid, stream)
+                             : launch_dtype<RPS_F32>(a, grid, topk_grid, stream);
 }
 
 cudaError_t row_stats_occupancy(int dtype, bool topk, int *blocks_per_sm) {

@@ -22,6 +22,25 @@ constexpr int kStatThreads = RPS_STAT_THREADS;  // ... and in statistics-only mo
 #endif
 constexpr int kStatBlocksPerSm = RPS_STAT_BLOCKS_PER_SM;
 __host__ __device__ constexpr int row_threads(bool topk) { return topk ? kRowThreads : kStatThreads; }
+#ifndef RPS_TOPK_SPLIT
+#define RPS_TOPK_SPLIT 1
+#endif
+constexpr bool kTopkSplit = RPS_TOPK_SPLIT != 0;  // top-k mode as a statistics launch plus a top-k launch
+#ifndef RPS_TOPK_WARPS
+#define RPS_TOPK_WARPS 4
+#endif
+#ifndef RPS_TOPK_MIN_BLOCKS
+#define RPS_TOPK_MIN_BLOCKS 4
+#endif
+constexpr int kTopkWarps = RPS_TOPK_WARPS;            // warps (rows in flight) per block of the top-k launch
+constexpr int kTopkMinBlocks = RPS_TOPK_MIN_BLOCKS;   // resident blocks per SM it is compiled for
+// Sketch entries per row slot: 32 per ring chunk of the row under the cut of
+// its statistics launch, at most units / 4 + 32 * kMaxPartials (at most
+// kMaxPartials pieces hold a part of a row, each may end in a partial chunk);
+// the fused top-k kernel indexes the sketch by unit instead.
+__host__ __device__ constexpr int64_t sketch_entries(int64_t units) {
+    return ((kTopkSplit ? (units + 3) / 4 + 32 * kMaxPartials : units) + 7) / 8 * 8;
+}
 // Shape of each warp's shared-memory ring (overridable at build time for tuning).
 #ifndef RPS_RING_UNITS_PER_LANE
 #define RPS_RING_UNITS_PER_LANE 4
@@ -69,7 +88,10 @@ struct RowStatsArgs {
     // workspace
     Partial *part;        // [slots][kMaxPartials]
     float2 *part_topk;    // [slots][kMaxPartials][k] as (value, index bits)
-    void *sketch;         // [slots][units_per_row] per-(chunk, lane) maxima (top-k mode)
+    void *sketch;         // [slots][sketch_stride] per-(chunk, lane) maxima (top-k mode)
+    int64_t sketch_stride;  // sketch entries per slot (a multiple of 8)
+    float4 *norm;         // [slots] B, ln S, 1 / S of each row's base-2 softmax and its sketch's len0 (top-k mode)
+    int32_t *sketch_piece;  // [1] units per piece of the sketch layout (top-k mode)
     uint32_t *ticket;     // [slots]
     // decomposition: the rows' 16-byte units are split evenly over `warps` warps
     int64_t units_per_row;
@@ -78,7 +100,9 @@ struct RowStatsArgs {
     uint32_t *err;
 };
 
-cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, cudaStream_t stream);
+// Top-k mode (a.k > 0) takes two launches: the statistics launch, which also
+// leaves the sketch and B, ln S, 1 / S, then the top-k launch of topk_grid blocks.
+cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, int topk_grid, cudaStream_t stream);
 cudaError_t row_stats_occupancy(int dtype, bool topk, int *blocks_per_sm);
 
 struct SelectArgs {

@@ -375,11 +375,12 @@ class Step:
 
     The base branch (0) of ``logits`` is the anchor, as in the workloads here.
     Kernels launched per ``run`` (one rps_run_step call): row statistics of the
-    masked base rows (top-k mode), pivot selection, row statistics of the
-    lookahead rows, and branch scores with the commit decision in one launch.
-    ``run_calls`` makes the same four launches through the separate calls.
+    masked base rows and their top-k lists (top-k mode: two launches), pivot
+    selection, row statistics of the lookahead rows, and branch scores with the
+    commit decision in one launch. ``run_calls`` makes the same five launches
+    through the separate calls.
     """
-    LAUNCHES = 4
+    LAUNCHES = 5
 
     def __init__(self, n_req: int, L: int, V: int, prm, device, dtype=torch.bfloat16):
         self.n_req, self.L, self.V, self.prm = n_req, L, V, prm
