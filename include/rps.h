@@ -216,6 +216,9 @@ rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream);
  * ties), and in top-k mode T_i (k_max tokens by logit desc / token asc),
  * mu = sum_{T_i} p_v and htrunc = -sum_{T_i} p_v log p_v (not renormalised).
  * fp32 arithmetic; argmax and T_i are exact (taken on the input values).
+ * Top-k mode makes two launches on `stream` (the statistics, then the top-k
+ * search over a sketch the first leaves in the workspace); statistics-only
+ * mode makes one.
  * Errors: RPS_ERR_INVALID_ARG for NULL pointers, a misaligned tensor, sizes out
  * of range or a workspace smaller than rps_workspace_bytes(n_seg * cap, vocab,
  * dtype, k); RPS_ERR_UNSUPPORTED above RPS_MAX_K / RPS_MAX_SEGMENTS.
@@ -288,7 +291,7 @@ rps_status rps_score_and_commit(const rps_logits *anchor_logits, int32_t anchor_
  * `base`, workspace d_ws_base), rps_select_pivots into `piv`, rps_score_step
  * over piv->branch_rows (statistics-only mode into `branch`, workspace
  * d_ws_branch, a different one), and rps_score_and_commit with branch 0 as the
- * anchor -- four launches with the results of the four calls. Every argument
+ * anchor -- five launches with the results of the four calls. Every argument
  * is checked before anything is enqueued. Because the call knows which launch
  * writes what, the select launch stages the mask before waiting for the base
  * statistics, and the score launch computes everything that does not read the
