@@ -19,7 +19,7 @@ constexpr size_t kAlign = 256;
 struct DeviceInfo {
     bool ready = false;
     int sm_count = 0;
-    int blocks[2][2] = {{0, 0}, {0, 0}};  // [dtype][topk]
+    int blocks[2] = {0, 0};  // resident row-statistics blocks per SM, by dtype
     uint32_t *err = nullptr;
 };
 
@@ -36,9 +36,7 @@ rps_status device_info(DeviceInfo *out) {
     if (!d.ready) {
         if (cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return RPS_ERR_CUDA;
         for (int dt = 0; dt < 2; ++dt)
-            for (int tk = 0; tk < 2; ++tk)
-                if (row_stats_occupancy(dt, tk != 0, &d.blocks[dt][tk]) != cudaSuccess || d.blocks[dt][tk] < 1)
-                    return RPS_ERR_CUDA;
+            if (row_stats_occupancy(dt, &d.blocks[dt]) != cudaSuccess || d.blocks[dt] < 1) return RPS_ERR_CUDA;
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return RPS_ERR_CUDA;
         d.err = static_cast<uint32_t *>(p);
@@ -84,12 +82,12 @@ rps_status check_logits(const rps_logits *l) {
 }
 
 struct WorkspaceLayout {
-    size_t ticket, part, topk, sketch, norm, piece, total;
+    size_t ticket, part, sketch, norm, piece, total;
 };
 
-// Tickets, partial records, per-piece top-k lists, the top-k sketch (one
-// element-sized entry per cell: one lane's units of one 2 KB ring chunk) and
-// each row's softmax reference and sum.
+// Tickets, partial records, and in top-k mode the sketch (one element-sized
+// entry per cell: one lane's units of one 2 KB ring chunk), each row's B, ln S,
+// 1 / S and first piece length, and the launch's piece length.
 WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k) {
     WorkspaceLayout w;
     const size_t rows = static_cast<size_t>(max_rows);
@@ -97,8 +95,7 @@ WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k
     const size_t units = (static_cast<size_t>(vocab) * esize + 15) / 16;
     w.ticket = 0;
     w.part = align_up(rows * sizeof(uint32_t));
-    w.topk = w.part + align_up(rows * kMaxPartials * sizeof(Partial));
-    w.sketch = w.topk + (k > 0 ? align_up(rows * kMaxPartials * static_cast<size_t>(k) * sizeof(float2)) : 0);
+    w.sketch = w.part + align_up(rows * kMaxPartials * sizeof(Partial));
     w.norm = w.sketch + (k > 0 ? align_up(rows * static_cast<size_t>(sketch_entries(units)) * esize) : 0);
     w.piece = w.norm + (k > 0 ? align_up(rows * sizeof(float4)) : 0);
     w.total = w.piece + (k > 0 ? align_up(sizeof(int32_t)) : 0);
@@ -193,16 +190,13 @@ rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows,
     char *ws = static_cast<char *>(d_ws);
     a.ticket = reinterpret_cast<uint32_t *>(ws + w.ticket);
     a.part = reinterpret_cast<Partial *>(ws + w.part);
-    a.part_topk = k > 0 ? reinterpret_cast<float2 *>(ws + w.topk) : nullptr;
     a.sketch = k > 0 ? static_cast<void *>(ws + w.sketch) : nullptr;
     a.norm = k > 0 ? reinterpret_cast<float4 *>(ws + w.norm) : nullptr;
     a.sketch_piece = k > 0 ? reinterpret_cast<int32_t *>(ws + w.piece) : nullptr;
     a.units_per_row = (logits->vocab + per_unit - 1) / per_unit;
     a.sketch_stride = sketch_entries(a.units_per_row);
-    // split top-k mode streams the rows with the statistics-only launch
-    const bool fused = topk && !kTopkSplit;
-    const int grid = dev.sm_count * dev.blocks[logits->dtype][fused ? 1 : 0];
-    a.warps = grid * (row_threads(fused) / 32);
+    const int grid = dev.sm_count * dev.blocks[logits->dtype];
+    a.warps = grid * (kStatThreads / 32);
     *topk_grid_out = static_cast<int>(std::min<int64_t>((max_rows + kTopkWarps - 1) / kTopkWarps,
                                                          static_cast<int64_t>(dev.sm_count) * 16));
     a.min_piece = (a.units_per_row + (kMaxPartials - 2) - 1) / (kMaxPartials - 2);

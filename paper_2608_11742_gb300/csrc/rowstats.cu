@@ -30,14 +30,14 @@
 // The exact maximum is tracked per unit; its token index is resolved once per
 // segment by re-reading the unit that holds it.
 //
-// Top-k (k <= 32, top-k mode only) takes a sketch and a short second pass. While
-// streaming, each lane records its maximum over its units of every ring chunk
-// (one value per 64 bytes of logits) in the workspace. After the segment, the
-// k-th largest of the 32 lane maxima is a lower bound on the segment's k-th
-// largest logit (those k lanes each hold an element at least that large); only
-// the (chunk, lane) pairs whose recorded maximum reaches the bound -- a handful --
-// are reloaded from L2, and their elements at or above it enter a warp-
-// distributed sorted list (lane j holds rank j in the order logit desc, token asc).
+// Top-k mode (k <= 32) is two launches. This one also records, per row, the
+// maximum of every cell -- one lane's four units of one ring chunk, 64 bytes of
+// logits 512 bytes apart -- densely in the workspace (the sketch), and the row's
+// B, ln S and 1 / S. topk_rows_kernel then takes one warp per row slot: the k-th
+// largest of its lanes' largest sketch entries bounds the row's k-th largest
+// logit from below (k lanes each saw a different cell holding an element at
+// least that large), so only the few cells that reach it are read again and
+// their elements at or above it merged into a warp-distributed sorted list.
 //
 // -inf logits or NaN make the first pass's sums NaN; the segment is then rescanned
 // from global memory with clamped exponents (SAFE), which scores -inf as
@@ -54,10 +54,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kSlack = 8.0f;          // nats the reference may trail the maximum
 constexpr int kChunkUnits = 32 * kBatch;  // 16-byte units per ring buffer (2 KB)
-// Staging area of the top-k second pass (top-k mode only): a lane's units of one
-// chunk, then the round's candidates, kCandBatch (value, token) pairs at a time.
-constexpr int kStageUnits = 32 * kBatch;
-constexpr int kCandBatch = 32;
+constexpr int kCandBatch = 32;  // top-k candidates merged at a time
 constexpr uint64_t kWaitLimitNs = 200ull * 1000 * 1000;  // a bulk copy normally lands within microseconds
 
 // ---------------------------------------------------------------- PTX helpers
@@ -262,9 +259,6 @@ struct LaneState {
     int best;         // unit (or first unit of the ring chunk) where mx was first reached, -1 if none
     bool best_chunk;  // best names a ring chunk: this lane's units best + 32 j, j < kBatch
     bool bad;         // NaN input seen (SAFE scan only)
-    float c1v, c2v;   // top-k mode: this lane's two largest chunk maxima ...
-    int c1u, c2u;     // ... and the first units of those chunks (-1 if none)
-    float c3v;        // top-k mode: its third largest chunk maximum (bounds every other chunk)
 };
 
 __device__ __forceinline__ void lane_init(LaneState &L) {
@@ -275,8 +269,6 @@ __device__ __forceinline__ void lane_init(LaneState &L) {
     L.best = -1;
     L.best_chunk = false;
     L.bad = false;
-    L.c1v = L.c2v = L.c3v = -INFINITY;
-    L.c1u = L.c2u = -1;
 }
 
 // Raise the exponent reference to m log2(e) (rare: only when m exceeds it by kSlack nats).
@@ -342,7 +334,7 @@ __device__ __forceinline__ void fold_unit(LaneState &L, const float (&y)[N], int
 // Fold this lane's units of one ring chunk (the fast path). The chunk's maximum
 // comes from packed compares; the exact argmax is resolved once per segment.
 // SKETCH: every lane records its maximum (-inf without units) at key + lane.
-template <int DT, bool TOPK, bool SKETCH>
+template <int DT, bool SKETCH>
 __device__ __forceinline__ float fold_chunk(LaneState &L, typename Elem<DT>::Sketch *sketch, const uint4 *buf,
                                             int n_units, int cu, int key, int lane) {
     using E = Elem<DT>;
@@ -359,23 +351,6 @@ __device__ __forceinline__ float fold_chunk(LaneState &L, typename Elem<DT>::Ske
     }
     raise_reference(L, cmax);
     if (SKETCH) sketch[key + lane] = E::to_sketch(cmax);
-    if (TOPK && j0_valid(n_units, lane)) {
-        sketch[cu + lane] = E::to_sketch(cmax);
-        if (cmax > L.c3v) {  // keep the three largest chunk maxima (first units of the top two)
-            L.c3v = fmaxf(L.c3v, fminf(cmax, L.c2v));
-        }
-        if (cmax > L.c2v) {
-            if (cmax > L.c1v) {
-                L.c2v = L.c1v;
-                L.c2u = L.c1u;
-                L.c1v = cmax;
-                L.c1u = cu;
-            } else {
-                L.c2v = cmax;
-                L.c2u = cu;
-            }
-        }
-    }
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
         if (j * 32 + lane < n_units) {
@@ -407,16 +382,7 @@ template <int DT>
 __device__ void rescan_safe(LaneState &L, const char *row, int V, int u0, int u1, int lane) {
     using E = Elem<DT>;
     constexpr int N = E::N;
-    // the top-k chunk record of the fast pass stays valid: -inf and NaN do not
-    // change a chunk's maximum
-    const float c1v = L.c1v, c2v = L.c2v, c3v = L.c3v;
-    const int c1u = L.c1u, c2u = L.c2u;
     lane_init(L);
-    L.c1v = c1v;
-    L.c2v = c2v;
-    L.c1u = c1u;
-    L.c2u = c2u;
-    L.c3v = c3v;
     const int full_end = min(u1, V / N);
     for (int u = u0 + lane; u < full_end; u += 32) {
         float y[N];
@@ -503,161 +469,6 @@ __device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, i
     }
 }
 
-// Second pass of a segment (top-k mode). theta is a lower bound on the segment's
-// k-th largest logit, so only the (chunk, lane) pairs whose recorded maximum
-// reaches it can hold a member of the top k.
-//
-// Bits j * N + i of the mask: element i of this lane's unit j of chunk cu
-// (staged at buf[j * 32 + lane]) is at or above th. Units are tested whole
-// first; most hold no such element.
-template <int DT>
-__device__ __forceinline__ unsigned long long cell_mask(const uint4 *buf, int cend, int cu, int lane, float th) {
-    using E = Elem<DT>;
-    constexpr int N = E::N;
-    unsigned long long cm = 0;
-    if (cu < 0) return 0;
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-        if (cu + j * 32 + lane < cend) {
-            const uint4 w = buf[j * 32 + lane];
-            if (E::unit_max(w) >= th) {
-                float y[N];
-                E::unpack(w, y);
-#pragma unroll
-                for (int i = 0; i < N; ++i)
-                    if (y[i] >= th) cm |= 1ull << (j * N + i);
-            }
-        }
-    }
-    return cm;
-}
-
-// Merges the elements at or above max(theta, current k-th entry) of up to two
-// staged chunks per lane (cu < 0: none) into the warp-distributed sorted list
-// (lane j = rank j), 32 at a time: the lanes compact their elements into the
-// candidate buffer, then warp_merge_batch. empty: the list holds nothing yet.
-template <int DT>
-__device__ __forceinline__ void topk_merge_cells(const uint4 *buf_a, int cu_a, const uint4 *buf_b, int cu_b, int cend,
-                                                 int k, int lane, float theta, float &tv, int &ti, float2 *cand,
-                                                 bool empty) {
-    using E = Elem<DT>;
-    constexpr int N = E::N;
-    constexpr int kCell = kBatch * N;
-    static_assert(2 * kCell <= 64, "candidate mask holds two chunks");
-    const float th = empty ? theta : fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
-    const unsigned long long cm =
-        cell_mask<DT>(buf_a, cend, cu_a, lane, th) | (cell_mask<DT>(buf_b, cend, cu_b, lane, th) << kCell);
-    const int c = __popc(static_cast<unsigned>(cm)) + __popc(static_cast<unsigned>(cm >> 32));
-    int incl = c;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int n = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += n;
-    }
-    const int total = __shfl_sync(kFull, incl, 31);
-    __syncwarp();
-    for (int done = 0; done < total; done += kCandBatch) {
-        // lanes write the candidates that fall in [done, done + kCandBatch)
-        int slot = incl - c;
-        unsigned long long bits = cm;
-        while (bits) {
-            const int bit = __ffsll(static_cast<long long>(bits)) - 1;
-            bits &= bits - 1;
-            if (slot >= done && slot < done + kCandBatch) {
-                const bool second = bit >= kCell;
-                const int e = second ? bit - kCell : bit;
-                const int j = e / N, i = e % N;
-                const uint32_t *words = reinterpret_cast<const uint32_t *>(second ? buf_b : buf_a);
-                const int cu = second ? cu_b : cu_a;
-                cand[slot - done] = make_float2(E::pick(words + (j * 32 + lane) * 4, i),
-                                                __int_as_float((cu + j * 32 + lane) * N + i));
-            }
-            ++slot;
-        }
-        __syncwarp();
-        const int idx = done + lane;
-        const float2 e = idx < total ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
-        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane, empty && done == 0);
-        __syncwarp();
-    }
-}
-
-// Stage this lane's units of chunk cu in buf by asynchronous 16-byte copies
-// (cu < 0: none); complete with cp_async_wait_all.
-__device__ __forceinline__ void stage_async(uint4 *buf, const char *row, int cend, int cu, int lane) {
-    if (cu < 0) return;
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-        const int u = cu + j * 32 + lane;
-        if (u < cend) cp_async16(buf + j * 32 + lane, row + static_cast<size_t>(u) * 16);
-    }
-}
-
-// A reload round: stage chunk cu (per lane) in stage, then merge.
-template <int DT>
-__device__ __forceinline__ void topk_round(const char *row, int cend, int cu, int k, int lane, float theta, float &tv,
-                                           int &ti, uint4 *stage, float2 *cand) {
-    __syncwarp();
-    stage_async(stage, row, cend, cu, lane);
-    cp_async_wait_all();
-    topk_merge_cells<DT>(stage, cu, stage, -1, cend, k, lane, theta, tv, ti, cand, false);
-}
-
-// ring2: two idle ring buffers (the warp's piece is fully streamed) or null.
-template <int DT>
-__device__ void topk_from_sketch(const LaneState &L, const char *row, const typename Elem<DT>::Sketch *sketch, int u0,
-                                 int cend, int k, int lane, float theta, float &tv, int &ti, uint4 *stage,
-                                 float2 *cand, uint4 *ring2) {
-    using E = Elem<DT>;
-    constexpr int kGroup = 16;  // recorded maxima a lane loads together
-    tv = -INFINITY;
-    ti = INT_MAX;
-    // Usually a lane's only chunks at or above the bound are its two best.
-    const int cu1 = L.c1v >= theta ? L.c1u : -1;
-    const int cu2 = L.c2v >= theta ? L.c2u : -1;
-    if (ring2) {
-        // both reloads in flight at once
-        __syncwarp();
-        stage_async(ring2, row, cend, cu1, lane);
-        stage_async(ring2 + kChunkUnits, row, cend, cu2, lane);
-        cp_async_wait_all();
-        topk_merge_cells<DT>(ring2, cu1, ring2 + kChunkUnits, cu2, cend, k, lane, theta, tv, ti, cand, true);
-    } else {
-        __syncwarp();
-        stage_async(stage, row, cend, cu1, lane);
-        cp_async_wait_all();
-        topk_merge_cells<DT>(stage, cu1, stage, -1, cend, k, lane, theta, tv, ti, cand, true);
-        if (__any_sync(kFull, cu2 >= 0)) topk_round<DT>(row, cend, cu2, k, lane, theta, tv, ti, stage, cand);
-    }
-    // Every other chunk of a lane peaks at most at its third largest chunk
-    // maximum: scan the recorded maxima only where that reaches the bound.
-    const bool more = L.c3v >= fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
-    if (!__any_sync(kFull, more)) return;
-    for (int c0 = u0; c0 < cend; c0 += kGroup * kChunkUnits) {
-        float m[kGroup];
-#pragma unroll
-        for (int g = 0; g < kGroup; ++g) {
-            const int key = c0 + g * kChunkUnits + lane;
-            m[g] = more && key < cend ? E::from_sketch(sketch[key]) : -INFINITY;
-        }
-        const float th0 = fmaxf(__shfl_sync(kFull, tv, k - 1), theta);
-        uint32_t hits = 0;
-#pragma unroll
-        for (int g = 0; g < kGroup; ++g) {
-            const int cu = c0 + g * kChunkUnits;
-            if (m[g] >= th0 && cu != L.c1u && cu != L.c2u) hits |= 1u << g;
-        }
-        while (__any_sync(kFull, hits != 0)) {
-            int cu = -1;
-            if (hits) {
-                cu = c0 + (__ffs(hits) - 1) * kChunkUnits;
-                hits &= hits - 1;
-            }
-            topk_round<DT>(row, cend, cu, k, lane, theta, tv, ti, stage, cand);
-        }
-    }
-}
-
 // Candidates of a row's ragged last unit (top-k mode).
 template <int DT>
 __device__ __forceinline__ void topk_tail(const char *row, int V, int k, int lane, float &tv, int &ti) {
@@ -741,9 +552,9 @@ __device__ __forceinline__ void topk_mass(float tv, float M, float lnS, float in
 
 // SKETCH: the row's B, ln S, 1 / S and sketch segment 0 (len0) are kept for
 // the top-k launch.
-template <bool SKETCH = false>
-__device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, const RowTotals &r, float tv, int ti,
-                                          int lane, int len0 = 0) {
+template <bool SKETCH>
+__device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, const RowTotals &r, int lane,
+                                          int len0) {
     const bool ok = (r.MX > -INFINITY) && (r.S > 0.f) && !(r.S != r.S) && !(r.T != r.T) && (r.AM != INT_MAX);
     // Probabilities are formed against the reference B like the sums, p_v =
     // 2^fma(z_v, log2(e), -B) / S, never as exp(z_v - lse): with large logits
@@ -766,61 +577,6 @@ __device__ __forceinline__ void write_row(const RowStatsArgs &a, int64_t slot, c
         if (!ok) flag_error(a.err, RPS_DEVERR_NONFINITE);
         if (SKETCH) a.norm[slot] = make_float4(r.M, lnS, invS, __int_as_float(len0));
     }
-    if (!SKETCH && a.k > 0) {
-        float mu, ht;
-        topk_mass(tv, r.M, lnS, invS, ok ? a.k : 0, lane, mu, ht);
-        if (lane == 0) {
-            a.mu[slot] = ok ? mu : NAN;
-            a.htrunc[slot] = ok ? ht : NAN;
-        }
-        if (lane < a.k) {
-            a.topk_idx[slot * a.k + lane] = ok ? ti : -1;
-            a.topk_logit[slot * a.k + lane] = ok ? tv : NAN;
-        }
-    }
-}
-
-// Merge of the top-k lists of every piece of a row (last arriver only). The
-// k-th largest list head bounds the row's k-th largest logit from below (k
-// lists each hold an element at least that large), so only the entries that
-// reach it are compacted into the candidate buffer and merged, 32 at a time.
-__device__ __forceinline__ void merge_topk(const float2 *lists, int count, int k, int lane, float &tv, int &ti,
-                                           float2 *cand) {
-    const int total = count * k;
-    const float head = lane < count ? __ldcg(&lists[lane * k].x) : -INFINITY;
-    const float bound = count >= k ? warp_kth_largest(head, k, lane) : -INFINITY;
-    tv = -INFINITY;
-    ti = INT_MAX;
-    int filled = 0;
-    bool empty = true;
-    auto flush = [&]() {
-        __syncwarp();
-        const float2 e = lane < filled ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
-        __syncwarp();
-        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane, empty);
-        empty = false;
-        filled = 0;
-    };
-    constexpr int kPer = 4;  // entries a lane loads together
-    for (int base = 0; base < total; base += 32 * kPer) {
-        float2 f[kPer];
-#pragma unroll
-        for (int q = 0; q < kPer; ++q) {
-            const int idx = base + q * 32 + lane;
-            f[q] = idx < total ? __ldcg(lists + idx) : make_float2(-INFINITY, __int_as_float(INT_MAX));
-        }
-#pragma unroll
-        for (int q = 0; q < kPer; ++q) {
-            const bool keep = base + q * 32 + lane < total && f[q].x >= bound;
-            const unsigned b = __ballot_sync(kFull, keep);
-            const int n = __popc(b);
-            if (n == 0) continue;
-            if (filled + n > 32) flush();
-            if (keep) cand[filled + __popc(b & ((1u << lane) - 1u))] = f[q];
-            filled += n;
-        }
-    }
-    if (filled > 0) flush();
 }
 
 // ---------------------------------------------------------------- segments
@@ -1038,18 +794,17 @@ struct Producer {
     }
 };
 
-// SKETCH (statistics-only, first launch of split top-k mode): also the sketch
-// (layout of sketch_row) and each row's B, ln S and 1 / S for the top-k launch.
-template <int DT, bool TOPK, bool SKETCH>
-__global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : kStatBlocksPerSm)
-    row_stats_kernel(const RowStatsArgs a) {
-    constexpr int kWarps = row_threads(TOPK) / 32;
+// SKETCH (first launch of top-k mode): also the sketch (layout of sketch_row)
+// and each row's B, ln S and 1 / S for the top-k launch.
+template <int DT, bool SKETCH>
+__global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kernel(const RowStatsArgs a) {
+    constexpr int kWarps = kStatThreads / 32;
     using E = Elem<DT>;
     constexpr int N = E::N;
     extern __shared__ __align__(128) uint4 dyn[];
     __shared__ int32_t seg_start[RPS_MAX_SEGMENTS + 1];
     __shared__ int32_t warp_total[kWarps];
-    constexpr int kRing = TOPK ? kStagesTopk : kStages;
+    constexpr int kRing = kStages;
     __shared__ __align__(8) uint64_t bars[kWarps][kRing];
 
     pdl_wait();
@@ -1057,12 +812,10 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
     const int lane = threadIdx.x & 31;
     const int wib = threadIdx.x >> 5;
     const int warp = blockIdx.x * kWarps + wib;
-    uint4 *ring = dyn + wib * (kRing * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0));
-    uint4 *stage = ring + kRing * kChunkUnits;  // top-k candidate staging (top-k mode only)
-    float2 *cand = reinterpret_cast<float2 *>(stage + kStageUnits);
+    uint4 *ring = dyn + wib * (kRing * kChunkUnits);
     uint64_t *bar = bars[wib];
 
-    const int64_t total_rows = count_rows<row_threads(TOPK)>(a, seg_start, warp_total, lane, wib);
+    const int64_t total_rows = count_rows<kStatThreads>(a, seg_start, warp_total, lane, wib);
 
     const int64_t nv = a.units_per_row;
     const int64_t total = total_rows * nv;
@@ -1070,13 +823,10 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
     // With at least as many warps as rows, each row is cut into equal pieces
     // (aligned: no piece crosses a row boundary, where a warp's stream would
     // stop for the row's record); otherwise the units are cut evenly.
-    // (statistics-only mode: the top-k launch keeps the even cut, whose index
-    // arithmetic its registers are tuned for)
-    __shared__ int64_t cut_cpr[TOPK ? 1 : kWarps];  // pieces per row of an aligned cut, 0 for the even cut
-    if (!TOPK && lane == 0) cut_cpr[wib] = 0;
+    __shared__ int64_t cut_cpr[kWarps];  // pieces per row of an aligned cut, 0 for the even cut
+    if (lane == 0) cut_cpr[wib] = 0;
     bool aligned = false;
-    const int64_t piece =
-        TOPK ? max((total + a.warps - 1) / a.warps, a.min_piece) : piece_units(a, total_rows, nv, aligned);
+    const int64_t piece = piece_units(a, total_rows, nv, aligned);
     if (SKETCH && blockIdx.x == 0 && threadIdx.x == 0) *a.sketch_piece = static_cast<int>(min(piece, nv));
     int64_t g_begin, g_end;
     if (aligned) {
@@ -1157,7 +907,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
         LaneState L;
         lane_init(L);
         typename E::Sketch *sketch =
-            TOPK || SKETCH ? static_cast<typename E::Sketch *>(a.sketch) + s.slot * a.sketch_stride : nullptr;
+            SKETCH ? static_cast<typename E::Sketch *>(a.sketch) + s.slot * a.sketch_stride : nullptr;
         const int cend = min(s.u1, full_units);
         int key = SKETCH ? sketch_key(sketch_row(sketch_len0(r, nv, piece, aligned), static_cast<int>(min(piece, nv)),
                                                  full_units),
@@ -1166,7 +916,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
         for (int cu = s.u0; cu < cend; cu += kChunkUnits) {
             int st;
             if (!acquire(st)) return;
-            fold_chunk<DT, TOPK, SKETCH>(L, sketch, ring + st * kChunkUnits, min(kChunkUnits, cend - cu), cu, key,
+            fold_chunk<DT, SKETCH>(L, sketch, ring + st * kChunkUnits, min(kChunkUnits, cend - cu), cu, key,
                                          lane);
             key += 32;
             release();
@@ -1188,36 +938,18 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
                 if (L.bad) L.s = pack2(NAN, NAN);
             }
         }
-        float tv = -INFINITY;
-        int ti = INT_MAX;
-        float seg_mx = L.mx;
-        int am;
-        if (TOPK) {
-            // the k-th largest lane maximum bounds the segment's k-th largest logit from below
-            // with nothing more in flight (the piece ends here) the ring stages the reloads
-            topk_from_sketch<DT>(L, s.row, sketch, s.u0, cend, a.k, lane, warp_kth_largest(L.mx, a.k, lane), tv, ti,
-                                 stage, cand, issued == acquired && kRing >= 2 ? ring : nullptr);
-            if (s.u1 > full_units) topk_tail<DT>(s.row, V, a.k, lane, tv, ti);
-            // rank 0 of T (largest logit, lowest token) is the argmax
-            const float t0 = __shfl_sync(kFull, tv, 0);
-            const int i0 = __shfl_sync(kFull, ti, 0);
-            seg_mx = lane == 0 ? t0 : -INFINITY;
-            am = lane == 0 ? i0 : INT_MAX;
-        } else if (SKETCH) {
-            am = 0;  // the top-k launch takes the argmax from its list
-        } else {
-            am = resolve_argmax<DT>(s.row, V, L, warp_max(L.mx), lane);
-        }
+        // (sketch mode: the top-k launch takes the argmax from its list)
+        const int am = SKETCH ? 0 : resolve_argmax<DT>(s.row, V, L, warp_max(L.mx), lane);
         float s_lo, s_hi, t_lo, t_hi;
         unpack2(L.s, s_lo, s_hi);
         unpack2(L.t, t_lo, t_hi);
-        RowTotals rt = combine(L.mref, s_lo + s_hi, t_lo + t_hi, seg_mx, am);
+        RowTotals rt = combine(L.mref, s_lo + s_hi, t_lo + t_hi, L.mx, am);
 
         // the pieces (warps) that hold a part of row r
         int64_t w_first;
         int count;
         // (read back from shared memory so that it is not kept live through the stream)
-        const int64_t cpr = TOPK ? 0 : *reinterpret_cast<volatile int64_t *>(&cut_cpr[TOPK ? 0 : wib]);
+        const int64_t cpr = *reinterpret_cast<volatile int64_t *>(&cut_cpr[wib]);
         if (cpr > 0) {
             w_first = r * cpr;
             count = static_cast<int>(cpr);
@@ -1227,7 +959,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
         }
         const int64_t slot = s.slot;
         if (count == 1) {
-            write_row<SKETCH>(a, slot, rt, tv, ti, lane, SKETCH ? sketch_len0(r, nv, piece, aligned) : 0);
+            write_row<SKETCH>(a, slot, rt, lane, SKETCH ? sketch_len0(r, nv, piece, aligned) : 0);
             continue;
         }
         const int my = static_cast<int>(warp - w_first);
@@ -1242,8 +974,6 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
             p.pad[0] = p.pad[1] = p.pad[2] = 0;
             part[my] = p;
         }
-        if (TOPK && lane < a.k)
-            a.part_topk[(slot * kMaxPartials + my) * a.k + lane] = make_float2(tv, __int_as_float(ti));
         __threadfence();
         __syncwarp();
         unsigned prior = 0;
@@ -1269,8 +999,7 @@ __global__ void __launch_bounds__(row_threads(TOPK), TOPK ? kTopkBlocksPerSm : k
             p.amax = __ldcg(&part[lane].amax);
         }
         rt = combine(p.mref, p.s, p.t, p.mx, p.amax);
-        if (TOPK) merge_topk(a.part_topk + slot * kMaxPartials * a.k, count, a.k, lane, tv, ti, cand);
-        write_row<SKETCH>(a, slot, rt, tv, ti, lane, SKETCH ? sketch_len0(r, nv, piece, aligned) : 0);
+        write_row<SKETCH>(a, slot, rt, lane, SKETCH ? sketch_len0(r, nv, piece, aligned) : 0);
     }
 }
 
@@ -1533,48 +1262,38 @@ __global__ void __launch_bounds__(kTopkWarps * 32, kTopkMinBlocks) topk_rows_ker
     }
 }
 
-template <int DT, bool TOPK>
-constexpr int dyn_smem_bytes() {
-    return row_threads(TOPK) / 32 * ((TOPK ? kStagesTopk : kStages) * kChunkUnits + (TOPK ? kStageUnits + kCandBatch / 2 : 0)) *
-           static_cast<int>(sizeof(uint4));
-}
+constexpr int kDynSmemBytes = kStatThreads / 32 * kStages * kChunkUnits * static_cast<int>(sizeof(uint4));
 
-template <int DT, bool TOPK, bool SKETCH = false>
+template <int DT, bool SKETCH>
 cudaError_t prepare_typed() {
-    return cudaFuncSetAttribute(row_stats_kernel<DT, TOPK, SKETCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                dyn_smem_bytes<DT, TOPK>());
+    return cudaFuncSetAttribute(row_stats_kernel<DT, SKETCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kDynSmemBytes);
 }
 
-template <int DT, bool TOPK, bool SKETCH = false>
+template <int DT, bool SKETCH>
 cudaError_t launch_typed(const RowStatsArgs &a, int grid, cudaStream_t stream) {
-    return launch_pdl(row_stats_kernel<DT, TOPK, SKETCH>, dim3(grid), dim3(row_threads(TOPK)),
-                      dyn_smem_bytes<DT, TOPK>(), stream, a);
+    return launch_pdl(row_stats_kernel<DT, SKETCH>, dim3(grid), dim3(kStatThreads), kDynSmemBytes, stream, a);
 }
 
-// Top-k mode as two launches: statistics with the sketch, then the top-k rows.
+// Statistics-only mode: one launch. Top-k mode: statistics with the sketch,
+// then the top-k rows.
 template <int DT>
-cudaError_t launch_split(const RowStatsArgs &a, int grid, int topk_grid, cudaStream_t stream) {
+cudaError_t launch_dtype(const RowStatsArgs &a, int grid, int topk_grid, cudaStream_t stream) {
+    if (a.k == 0) return launch_typed<DT, false>(a, grid, stream);
     RowStatsArgs st = a;
     st.k = 0;
-    cudaError_t e = launch_typed<DT, false, true>(st, grid, stream);
+    cudaError_t e = launch_typed<DT, true>(st, grid, stream);
     if (e != cudaSuccess) return e;
     return launch_pdl(topk_rows_kernel<DT>, dim3(topk_grid), dim3(kTopkWarps * 32), 0, stream, a);
 }
 
-template <int DT, bool TOPK>
-cudaError_t occupancy_typed(int *blocks) {
-    cudaError_t e = prepare_typed<DT, TOPK>();
-    if (e != cudaSuccess) return e;
-    if (!TOPK && (e = prepare_typed<DT, false, true>()) != cudaSuccess) return e;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, TOPK, false>, row_threads(TOPK),
-                                                         dyn_smem_bytes<DT, TOPK>());
-}
-
 template <int DT>
-cudaError_t launch_dtype(const RowStatsArgs &a, int grid, int topk_grid, cudaStream_t stream) {
-    if (a.k == 0) return launch_typed<DT, false>(a, grid, stream);
-    if (kTopkSplit) return launch_split<DT>(a, grid, topk_grid, stream);
-    return launch_typed<DT, true>(a, grid, stream);
+cudaError_t occupancy_typed(int *blocks) {
+    cudaError_t e = prepare_typed<DT, false>();
+    if (e == cudaSuccess) e = prepare_typed<DT, true>();
+    if (e != cudaSuccess) return e;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, row_stats_kernel<DT, false>, kStatThreads,
+                                                         kDynSmemBytes);
 }
 
 }  // namespace
@@ -1584,10 +1303,8 @@ cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, int top
                              : launch_dtype<RPS_F32>(a, grid, topk_grid, stream);
 }
 
-cudaError_t row_stats_occupancy(int dtype, bool topk, int *blocks_per_sm) {
-    if (dtype == RPS_BF16) return topk ? occupancy_typed<RPS_BF16, true>(blocks_per_sm)
-                                       : occupancy_typed<RPS_BF16, false>(blocks_per_sm);
-    return topk ? occupancy_typed<RPS_F32, true>(blocks_per_sm) : occupancy_typed<RPS_F32, false>(blocks_per_sm);
+cudaError_t row_stats_occupancy(int dtype, int *blocks_per_sm) {
+    return dtype == RPS_BF16 ? occupancy_typed<RPS_BF16>(blocks_per_sm) : occupancy_typed<RPS_F32>(blocks_per_sm);
 }
 
 }  // namespace rps

@@ -12,20 +12,14 @@ namespace rps {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kMaxPartials = 32;   // partial records per row (one merging warp)
-constexpr int kRowThreads = 256;   // threads per block of the row-statistics kernel in top-k mode
 #ifndef RPS_STAT_THREADS
 #define RPS_STAT_THREADS 1024
 #endif
-constexpr int kStatThreads = RPS_STAT_THREADS;  // ... and in statistics-only mode (one block per SM: no launch-slot skew)
+constexpr int kStatThreads = RPS_STAT_THREADS;  // threads per block of the row-statistics kernel (one block per SM: no launch-slot skew)
 #ifndef RPS_STAT_BLOCKS_PER_SM
 #define RPS_STAT_BLOCKS_PER_SM 1
 #endif
 constexpr int kStatBlocksPerSm = RPS_STAT_BLOCKS_PER_SM;
-__host__ __device__ constexpr int row_threads(bool topk) { return topk ? kRowThreads : kStatThreads; }
-#ifndef RPS_TOPK_SPLIT
-#define RPS_TOPK_SPLIT 1
-#endif
-constexpr bool kTopkSplit = RPS_TOPK_SPLIT != 0;  // top-k mode as a statistics launch plus a top-k launch
 #ifndef RPS_TOPK_WARPS
 #define RPS_TOPK_WARPS 4
 #endif
@@ -36,10 +30,9 @@ constexpr int kTopkWarps = RPS_TOPK_WARPS;            // warps (rows in flight) 
 constexpr int kTopkMinBlocks = RPS_TOPK_MIN_BLOCKS;   // resident blocks per SM it is compiled for
 // Sketch entries per row slot: 32 per ring chunk of the row under the cut of
 // its statistics launch, at most units / 4 + 32 * kMaxPartials (at most
-// kMaxPartials pieces hold a part of a row, each may end in a partial chunk);
-// the fused top-k kernel indexes the sketch by unit instead.
+// kMaxPartials pieces hold a part of a row, each may end in a partial chunk).
 __host__ __device__ constexpr int64_t sketch_entries(int64_t units) {
-    return ((kTopkSplit ? (units + 3) / 4 + 32 * kMaxPartials : units) + 7) / 8 * 8;
+    return ((units + 3) / 4 + 32 * kMaxPartials + 7) / 8 * 8;
 }
 // Shape of each warp's shared-memory ring (overridable at build time for tuning).
 #ifndef RPS_RING_UNITS_PER_LANE
@@ -50,14 +43,6 @@ __host__ __device__ constexpr int64_t sketch_entries(int64_t units) {
 #endif
 constexpr int kBatch = RPS_RING_UNITS_PER_LANE;  // 16-byte units a lane takes from each ring buffer
 constexpr int kStages = RPS_RING_STAGES;         // ring buffers (bulk copies in flight) per warp
-#ifndef RPS_RING_STAGES_TOPK
-#define RPS_RING_STAGES_TOPK RPS_RING_STAGES
-#endif
-#ifndef RPS_TOPK_BLOCKS_PER_SM
-#define RPS_TOPK_BLOCKS_PER_SM 4
-#endif
-constexpr int kStagesTopk = RPS_RING_STAGES_TOPK;     // ring buffers per warp in top-k mode
-constexpr int kTopkBlocksPerSm = RPS_TOPK_BLOCKS_PER_SM;  // resident blocks the top-k kernel is compiled for
 
 // Partial statistics of one row segment, base-2 online softmax:
 // s = sum 2^u, t = sum u 2^u with u = (z - mref) * log2(e); mx = max z and
@@ -87,7 +72,6 @@ struct RowStatsArgs {
     int32_t *argmax, *topk_idx;
     // workspace
     Partial *part;        // [slots][kMaxPartials]
-    float2 *part_topk;    // [slots][kMaxPartials][k] as (value, index bits)
     void *sketch;         // [slots][sketch_stride] per-(chunk, lane) maxima (top-k mode)
     int64_t sketch_stride;  // sketch entries per slot (a multiple of 8)
     float4 *norm;         // [slots] B, ln S, 1 / S of each row's base-2 softmax and its sketch's len0 (top-k mode)
@@ -103,7 +87,7 @@ struct RowStatsArgs {
 // Top-k mode (a.k > 0) takes two launches: the statistics launch, which also
 // leaves the sketch and B, ln S, 1 / S, then the top-k launch of topk_grid blocks.
 cudaError_t launch_row_stats(const RowStatsArgs &a, int dtype, int grid, int topk_grid, cudaStream_t stream);
-cudaError_t row_stats_occupancy(int dtype, bool topk, int *blocks_per_sm);
+cudaError_t row_stats_occupancy(int dtype, int *blocks_per_sm);
 
 struct SelectArgs {
     // base statistics [q * L + k]

@@ -93,6 +93,7 @@ ROW_CASES = [
     ("f32", 1001, 64, 1),
     ("bf16", 126464, 3, 10),     # few long rows: each split over many warps
     ("bf16", 151936, 2, 16),
+    ("f32", 126464, 3, 10),      # a sketch longer than one batch of loads per lane
     ("bf16", 40, 33, 32),        # rows shorter than one batch
     ("f32", 17, 5, 17),          # k == V
 ]
@@ -185,6 +186,62 @@ def test_device_errors_are_reported(rps):
     rps.rps_score_step(to_device(z), None, cnt, 1, 4, Params(), buf4, ws4, mask_pos=mpos)
     status, detail = rps.rps_poll_device_status()
     assert status == rps.RPS_ERR_DEVICE and detail & rps.DEVERR_MASK
+
+
+def test_topk_rows_with_few_finite_logits(rps):
+    """Rows with fewer finite logits than k (the top-k bound is -inf, so every cell,
+    the sketch's -inf padding included, is a candidate, and the list fills with -inf
+    entries in token order) and with a few more, in top-k mode."""
+    for dtype, V, k in (("bf16", 5003, 10), ("f32", 2049, 32)):
+        rng = np.random.default_rng(V + k)
+        counts = [1, 3, k - 1, k, k + 1, 40]
+        rows = np.full((len(counts), V), -np.inf, np.float32)
+        for i, c in enumerate(counts):
+            rows[i, rng.choice(V, c, replace=False)] = rng.standard_normal(c).astype(np.float32) * np.float32(3.0)
+        if dtype == "bf16":
+            rows = synth.bf16_round(rows)
+        n = len(counts)
+        t = padded_tensor(rows.reshape(1, 1, n, V))
+        ref = oracle_default().row_stats(rows, k)
+        desc = torch.tensor([[0, 0, i] for i in range(n)], dtype=torch.int32, device="cuda")
+        buf = rps.RowStatsBuf.alloc(n, k, "cuda")
+        ws = torch.zeros(rps.rps_workspace_bytes(n, V, k, t.dtype), dtype=torch.uint8, device="cuda")
+        rps.rps_score_step(t, desc, None, 1, n, Params(k_max=k), buf, ws)
+        status, detail = rps.rps_poll_device_status()
+        assert status == rps.RPS_OK, hex(detail)
+        compare_stats(stats_np(buf), ref, np.arange(n), k, f"{dtype} V={V} few finite")
+
+
+def test_topk_mode_device_errors(rps):
+    """Top-k mode: a NaN row gives NaN statistics, an empty list and argmax -1; a bad
+    descriptor leaves its slot untouched; a mask count above capacity is clamped."""
+    V, k = 3001, 8
+    rng = np.random.default_rng(11)
+    z = rng.standard_normal((1, 1, 4, V)).astype(np.float32)
+    z[0, 0, 2, 7] = np.nan
+    t = padded_tensor(z)
+    buf = rps.RowStatsBuf.alloc(3, k, "cuda")
+    ws = torch.zeros(rps.rps_workspace_bytes(3, V, k, t.dtype), dtype=torch.uint8, device="cuda")
+    desc = torch.tensor([[0, 0, 0], [0, 0, 9], [0, 0, 2]], dtype=torch.int32, device="cuda")  # pos 9 out of range
+    rps.rps_score_step(t, desc, None, 1, 3, Params(k_max=k), buf, ws)
+    status, detail = rps.rps_poll_device_status()
+    assert status == rps.RPS_ERR_DEVICE
+    assert detail & rps.DEVERR_ROW_INDEX and detail & rps.DEVERR_NONFINITE
+    g = stats_np(buf)
+    compare_stats(g, oracle_default().row_stats(z[0, 0, :1], k), [0], k, "finite row")
+    assert np.isnan(g.H[1]) and g.argmax[1] == -1 and (g.topk_idx[1] == -1).all(), "bad descriptor: untouched"
+    assert np.isnan(g.H[2]) and g.argmax[2] == -1 and np.isnan(g.mu[2]) and np.isnan(g.htrunc[2])
+    assert (g.topk_idx[2] == -1).all() and np.isnan(g.topk_logit[2]).all()
+    # a mask count above capacity is clamped (all four rows scored) and flagged
+    z[0, 0, 2, 7] = 0.0
+    cnt = torch.tensor([9], dtype=torch.int32, device="cuda")
+    mpos = torch.arange(4, dtype=torch.int32, device="cuda").view(1, 4)
+    buf4 = rps.RowStatsBuf.alloc(4, k, "cuda")
+    ws4 = torch.zeros(rps.rps_workspace_bytes(4, V, k, torch.float32), dtype=torch.uint8, device="cuda")
+    rps.rps_score_step(padded_tensor(z), None, cnt, 1, 4, Params(k_max=k), buf4, ws4, mask_pos=mpos)
+    status, detail = rps.rps_poll_device_status()
+    assert status == rps.RPS_ERR_DEVICE and detail & rps.DEVERR_MASK
+    compare_stats(stats_np(buf4), oracle_default().row_stats(z[0, 0], k), np.arange(4), k, "clamped count")
 
 
 # ----------------------------------------------------------------------------- full steps
