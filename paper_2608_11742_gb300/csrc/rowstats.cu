@@ -610,8 +610,16 @@ __device__ __forceinline__ int64_t count_rows(const RowStatsArgs &a, int32_t *se
     }
     if (lane == 31) warp_total[wib] = incl;
     __syncthreads();
-    int32_t run = incl - local;
-    for (int w = 0; w < wib; ++w) run += warp_total[w];
+    // exclusive prefix of the warps' totals: a shuffle scan in every warp
+    static_assert(THREADS <= 32 * 32, "one warp scans the warps' totals");
+    const int32_t wt = lane < THREADS / 32 ? warp_total[lane] : 0;
+    int32_t wincl = wt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t n = __shfl_up_sync(kFull, wincl, o);
+        if (lane >= o) wincl += n;
+    }
+    int32_t run = __shfl_sync(kFull, wincl - wt, wib) + incl - local;
 #pragma unroll
     for (int i = 0; i < kPer; ++i) {
         seg_start[threadIdx.x * kPer + i] = run;
@@ -682,11 +690,12 @@ __device__ __forceinline__ void locate(const RowStatsArgs &a, const int32_t *seg
 __device__ __forceinline__ int64_t piece_units(const RowStatsArgs &a, int64_t total_rows, int64_t nv,
                                                bool &aligned) {
     aligned = false;
-    if (total_rows <= a.warps) {
-        const int64_t ppr = min(static_cast<int64_t>(a.warps) / total_rows, (nv + a.min_piece - 1) / a.min_piece);
-        const int64_t piece = (nv + ppr - 1) / ppr;
-        const int64_t cpr = (nv + piece - 1) / piece;
-        if (8 * total_rows * cpr >= 7 * static_cast<int64_t>(a.warps)) {
+    if (total_rows <= a.warps) {  // 32-bit arithmetic: rows, warps and units of a row fit
+        const int rows = static_cast<int>(total_rows), n = static_cast<int>(nv), mp = static_cast<int>(a.min_piece);
+        const int ppr = min(a.warps / rows, (n + mp - 1) / mp);
+        const int piece = (n + ppr - 1) / ppr;
+        const int cpr = (n + piece - 1) / piece;
+        if (8 * static_cast<int64_t>(rows) * cpr >= 7 * static_cast<int64_t>(a.warps)) {
             aligned = true;
             return piece;
         }
@@ -747,15 +756,24 @@ __device__ __forceinline__ void sketch_cell(const SketchRow &q, int full_units, 
     count = first < end ? min((end - first + 31) / 32, kBatch) : 0;
 }
 
-// Walks the row segments of the global unit range [g, g_end).
+// A warp's unit range: `left` units from unit u of row r on.
+struct Walk {
+    int64_t r;
+    int u;
+    int64_t left;
+};
+
+// Walks the row segments of a warp's range.
 template <int DT>
-__device__ __forceinline__ bool next_segment(const RowStatsArgs &a, const int32_t *seg_start, int64_t nv, int64_t &g,
-                                             int64_t g_end, int64_t &r, Segment &s) {
-    if (g >= g_end) return false;
-    r = g / nv;
-    s.u0 = static_cast<int>(g - r * nv);
-    s.u1 = static_cast<int>(min(nv, static_cast<int64_t>(s.u0) + (g_end - g)));
-    g += s.u1 - s.u0;
+__device__ __forceinline__ bool next_segment(const RowStatsArgs &a, const int32_t *seg_start, int64_t nv, Walk &w,
+                                             int64_t &r, Segment &s) {
+    if (w.left <= 0) return false;
+    r = w.r;
+    s.u0 = w.u;
+    s.u1 = static_cast<int>(min(nv, static_cast<int64_t>(w.u) + w.left));
+    w.left -= s.u1 - s.u0;
+    ++w.r;
+    w.u = 0;
     locate<DT>(a, seg_start, r, s);
     return true;
 }
@@ -764,15 +782,14 @@ __device__ __forceinline__ bool next_segment(const RowStatsArgs &a, const int32_
 // piece, in the order the warp consumes them (valid segments only).
 template <int DT>
 struct Producer {
-    int64_t g, g_end;
+    Walk w;
     Segment s;
     int cu;      // next unit to copy in the current segment
     int cu_end;  // end of its whole units
     bool have;
 
-    __device__ __forceinline__ void init(int64_t g0, int64_t g1) {
-        g = g0;
-        g_end = g1;
+    __device__ __forceinline__ void init(const Walk &w0) {
+        w = w0;
         have = false;
         cu = cu_end = 0;
     }
@@ -781,7 +798,7 @@ struct Producer {
                                          const char *&src, uint32_t &bytes) {
         while (!have || cu >= cu_end) {
             int64_t r;
-            if (!next_segment<DT>(a, seg_start, nv, g, g_end, r, s)) return false;
+            if (!next_segment<DT>(a, seg_start, nv, w, r, s)) return false;
             have = s.valid;
             cu = s.u0;
             cu_end = min(s.u1, full_units);
@@ -828,18 +845,21 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
     bool aligned = false;
     const int64_t piece = piece_units(a, total_rows, nv, aligned);
     if (SKETCH && blockIdx.x == 0 && threadIdx.x == 0) *a.sketch_piece = static_cast<int>(min(piece, nv));
-    int64_t g_begin, g_end;
-    if (aligned) {
-        const int64_t cpr = (nv + piece - 1) / piece;  // pieces per row
-        const int64_t row0 = warp / cpr, part = warp % cpr;
+    Walk w0;
+    if (aligned) {  // (32-bit: piece and the pieces per row are below the row length)
+        const int cpr = (static_cast<int>(nv) + static_cast<int>(piece) - 1) / static_cast<int>(piece);
+        const int row0 = warp / cpr, part = warp - row0 * cpr;
         if (row0 >= total_rows) return;
-        g_begin = row0 * nv + part * piece;
-        g_end = min(g_begin + piece, (row0 + 1) * nv);
+        w0.r = row0;
+        w0.u = part * static_cast<int>(piece);
+        w0.left = min(piece, nv - w0.u);
         if (lane == 0) cut_cpr[wib] = cpr;
     } else {
-        g_begin = static_cast<int64_t>(warp) * piece;
+        const int64_t g_begin = static_cast<int64_t>(warp) * piece;
         if (g_begin >= total) return;
-        g_end = min(g_begin + piece, total);
+        w0.r = g_begin / nv;
+        w0.u = static_cast<int>(g_begin - w0.r * nv);
+        w0.left = min(piece, total - g_begin);
     }
     const int V = static_cast<int>(a.vocab);
     const int full_units = V / N;
@@ -851,7 +871,7 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
     }
     __syncwarp();
     Producer<DT> prod;
-    prod.init(g_begin, g_end);
+    prod.init(w0);
     int issued = 0;
     if (lane == 0) {
         const char *src;
@@ -896,10 +916,10 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
         issued = __shfl_sync(kFull, issued, 0);
     };
 
-    int64_t g = g_begin;
+    Walk walk = w0;
     int64_t r;
     Segment s;
-    while (next_segment<DT>(a, seg_start, nv, g, g_end, r, s)) {
+    while (next_segment<DT>(a, seg_start, nv, walk, r, s)) {
         if (!s.valid) {
             if (s.bad && lane == 0) flag_error(a.err, RPS_DEVERR_ROW_INDEX);
             continue;
