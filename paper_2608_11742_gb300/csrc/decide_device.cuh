@@ -94,27 +94,29 @@ __device__ __forceinline__ uint64_t pivot_key(float v, int pos) {
 }
 
 // The P <= RPS_MAX_PIVOTS largest of n distinct keys (0 = none), into out[0..P)
-// in descending order: in every group of 32, each key counts the larger keys of
-// its group and the best P move on, until one group is left. Every level at
-// least halves n - P, so a level's output fits t_a / t_b of n / 2 + 32 keys; the
-// level cap forces the last level all the same.
+// in descending order: in every group of 32 (one warp, a key per lane), each
+// key counts the larger keys of its group by shuffles and the best P move on,
+// until one group is left. With P <= 16 a level takes n to at most n / 2 + 16,
+// so the levels end and each one's output fits t_a / t_b of n / 2 + 32 keys.
+static_assert(RPS_MAX_PIVOTS <= 16 && RPS_MAX_COMMIT_K <= 16, "block_top_keys halves the keys per level");
 __device__ void block_top_keys(const uint64_t *keys, int n, int P, uint64_t *t_a, uint64_t *t_b, uint64_t *out) {
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31;
     const uint64_t *cur = keys;
     uint64_t *nxt = t_a;
-    for (int level = 0;; ++level) {
-        const int groups = level == 11 ? 1 : (n + 31) / 32;
+    for (;;) {
+        const int groups = (n + 31) / 32;
         uint64_t *dst = groups <= 1 ? out : nxt;
         const int n_dst = groups <= 1 ? P : groups * P;
         for (int t = tid; t < n_dst; t += blockDim.x) dst[t] = 0ull;
         __syncthreads();
-        for (int t = tid; t < n; t += blockDim.x) {
-            const uint64_t me = cur[t];
-            if (me == 0ull) continue;
-            const int g0 = groups <= 1 ? 0 : t & ~31, g1 = groups <= 1 ? n : min(n, g0 + 32);
+        // (blockDim.x is a multiple of 32: a warp's lanes hold one whole group)
+        for (int t0 = tid & ~31; t0 < n; t0 += blockDim.x) {
+            const int t = t0 + lane;
+            const uint64_t me = t < n ? cur[t] : 0ull;
             int rank = 0;
-            for (int u = g0; u < g1; ++u) rank += cur[u] > me;
-            if (rank < P) dst[(groups <= 1 ? 0 : (t >> 5) * P) + rank] = me;
+#pragma unroll
+            for (int u = 0; u < 32; ++u) rank += __shfl_sync(kFull, me, u) > me;
+            if (me != 0ull && rank < P) dst[(groups <= 1 ? 0 : (t0 >> 5) * P) + rank] = me;
         }
         __syncthreads();
         if (groups <= 1) return;
@@ -396,12 +398,13 @@ __device__ void select_request(const SelectArgs &a, int q, unsigned char *smem, 
             const int b = valid_b[m];
             const int pi = piv_i[b / K];
             int32_t *rows = o.branch_rows + (static_cast<int64_t>(q) * NB * L + br_off[b]) * 3;
-            // the (q, 1 + b, pos) triples as consecutive words: contiguous stores
-            const int n_words = (n_rem - 1) * 3;
-            for (int x = lane; x < n_words; x += 32) {
-                const int d = x / 3, f = x - d * 3;
+            // the (q, 1 + b, pos) triples, one per lane: the warp's three stores
+            // cover 384 consecutive bytes
+            for (int d = lane; d < n_rem - 1; d += 32) {
                 const int i = d < pi ? d : d + 1;
-                rows[x] = f == 0 ? q : f == 1 ? 1 + b : rp[i];
+                rows[3 * d] = q;
+                rows[3 * d + 1] = 1 + b;
+                rows[3 * d + 2] = rp[i];
             }
         }
     }
