@@ -533,9 +533,23 @@ __device__ void score_finish(const ScoreArgs &a, int q, const PivotView &v, cons
                 const int b = j * K + c;
                 const int64_t first = static_cast<int64_t>(q) * NB * L + v.branch_off[b];
                 const int n = v.branch_cnt[b];
-                for (int i = lane; i < n; i += 32) {
-                    sum += __ldcg(a.b_H + first + i);
-                    count += __ldcg(a.b_pmax + first + i) >= a.tau;
+                // lane's entries lane + 32 t in order; eight at a time in flight
+                constexpr int kIn = 8;
+                for (int i0 = 0; i0 < n; i0 += 32 * kIn) {
+                    float h[kIn], pm[kIn];
+#pragma unroll
+                    for (int u = 0; u < kIn; ++u) {
+                        const int i = i0 + u * 32 + lane;
+                        h[u] = i < n ? __ldcg(a.b_H + first + i) : 0.f;
+                        pm[u] = i < n ? __ldcg(a.b_pmax + first + i) : 0.f;
+                    }
+#pragma unroll
+                    for (int u = 0; u < kIn; ++u) {
+                        if (i0 + u * 32 + lane < n) {
+                            sum += h[u];
+                            count += pm[u] >= a.tau;
+                        }
+                    }
                 }
                 sum = warp_sum(sum);
                 count = warp_sum_int(count);
