@@ -4,12 +4,14 @@
 //   zmax, argmax (Eq. 1), lse, H = -sum p log p, P^max (Sec. 2 notation) and,
 //   in top-k mode, T_i, mu_i and the truncated entropy of Eq. 3.
 //
-// Work split. The rows' 16-byte units are laid end to end and cut into equal
-// contiguous pieces, one per warp of a persistent grid, so every warp streams
-// the same number of bytes whatever the row count. A piece covers the tail of
-// one row, whole rows and the head of another; each (warp, row) pair leaves a
-// partial record in the workspace and the last warp to finish a row (atomic
-// ticket, no waiting) merges the at most kMaxPartials records and writes the row.
+// Work split. One block of kStatThreads per SM; each warp streams one piece. With
+// at least as many warps as rows, each row is cut into equal pieces, so that no
+// piece crosses a row boundary; otherwise the rows' 16-byte units are laid end
+// to end and cut into equal contiguous pieces (a piece covers the tail of one
+// row, whole rows and the head of another). Either way every warp streams about
+// the same number of bytes. Each (warp, row) pair leaves a partial record in the
+// workspace and the last warp to finish a row (atomic ticket, no waiting) merges
+// the at most kMaxPartials records and writes the row.
 //
 // Data movement. Each warp owns a ring of shared-memory buffers of 2 KB.
 // Lane 0 keeps every free buffer filled by a bulk asynchronous copy (cp.async.bulk, completion
@@ -28,7 +30,8 @@
 // and P^max, mu and the truncated entropy take their exponents the same way, so
 // a rounding of B is a common factor of numerator and denominator.
 // The exact maximum is tracked per unit; its token index is resolved once per
-// segment by re-reading the unit that holds it.
+// segment by re-reading the unit that holds it (in top-k mode it is rank 0 of
+// the top-k list instead).
 //
 // Top-k mode (k <= 32) is two launches. This one also records, per row, the
 // maximum of every cell -- one lane's four units of one ring chunk, 64 bytes of
