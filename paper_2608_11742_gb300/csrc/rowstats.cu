@@ -445,18 +445,36 @@ __device__ __forceinline__ void pair_step(float &v, int &i, int stride, bool kee
     }
 }
 
-__device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, int ci, int k, int lane,
-                                                 bool empty = false) {
+// The list holds nothing yet: each real candidate's rank among the 32 is the
+// count of candidates before it (candidates are distinct, so ranks are); ranks
+// below k go to buf[rank] (kCandBatch entries), then lane j takes rank j.
+// Independent shuffles instead of a sorting network's dependent stages.
+__device__ __forceinline__ void warp_rank_into_list(float &tv, int &ti, float cv, int ci, int k, int lane,
+                                                    float2 *buf) {
+    const bool real = ci != INT_MAX;
+    int rank = 0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        const float ov = __shfl_sync(kFull, cv, j);
+        const int oi = __shfl_sync(kFull, ci, j);
+        rank += ranks_before(ov, oi, cv, ci);
+    }
+    const int n = __popc(__ballot_sync(kFull, real));
+    __syncwarp();
+    if (real && rank < k) buf[rank] = make_float2(cv, __int_as_float(ci));
+    __syncwarp();
+    const float2 e = lane < k && lane < n ? buf[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
+    tv = e.x;
+    ti = __float_as_int(e.y);
+    __syncwarp();
+}
+
+__device__ __forceinline__ void warp_merge_batch(float &tv, int &ti, float cv, int ci, int k, int lane) {
 #pragma unroll
     for (int size = 2; size <= 32; size <<= 1) {
 #pragma unroll
         for (int stride = size >> 1; stride > 0; stride >>= 1)
             pair_step(cv, ci, stride, ((lane & size) == 0) == ((lane & stride) == 0));
-    }
-    if (empty) {  // the list held nothing: the sorted candidates are the list
-        tv = lane < k ? cv : -INFINITY;
-        ti = lane < k ? ci : INT_MAX;
-        return;
     }
     const float rv = __shfl_sync(kFull, cv, 31 - lane);
     const int ri = __shfl_sync(kFull, ci, 31 - lane);
@@ -590,6 +608,19 @@ template <int THREADS>
 __device__ __forceinline__ int64_t count_rows(const RowStatsArgs &a, int32_t *seg_start, int32_t *warp_total, int lane,
                                               int wib) {
     if (!a.seg_cnt) return static_cast<int64_t>(a.n_seg) * a.cap;
+    if (a.n_seg == 1) {  // one request: no scan (locate reads seg_start[0] only)
+        int32_t v = a.seg_cnt[0];
+        if (v < 0 || v > a.cap) {
+            if (blockIdx.x == 0 && threadIdx.x == 0) flag_error(a.err, RPS_DEVERR_MASK);
+            v = v < 0 ? 0 : a.cap;
+        }
+        if (threadIdx.x == 0) {
+            seg_start[0] = 0;
+            seg_start[1] = v;
+        }
+        __syncthreads();
+        return v;
+    }
     constexpr int kPer = RPS_MAX_SEGMENTS / THREADS;
     static_assert(RPS_MAX_SEGMENTS % THREADS == 0, "segments split evenly over the threads");
     int32_t c[kPer];
@@ -1086,7 +1117,9 @@ __device__ __forceinline__ void merge_staged_cells(const uint4 *stage, int first
         }
         __syncwarp();
         const float2 e = done + lane < total ? cand[lane] : make_float2(-INFINITY, __int_as_float(INT_MAX));
-        warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane, empty);
+        __syncwarp();
+        if (empty) warp_rank_into_list(tv, ti, e.x, __float_as_int(e.y), k, lane, cand);
+        else warp_merge_batch(tv, ti, e.x, __float_as_int(e.y), k, lane);
         empty = false;
         __syncwarp();
     }
