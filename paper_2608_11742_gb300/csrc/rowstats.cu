@@ -1235,7 +1235,11 @@ __global__ void __launch_bounds__(kTopkWarps * 32, kTopkMinBlocks) topk_rows_ker
             }
             continue;
         }
-        const SketchRow cut = sketch_row(__float_as_int(nrm.w), piece, full_units);
+        // (clamped: a record or a piece length left by a failed launch never
+        // names a unit outside the row)
+        const int n_units = static_cast<int>(nv);
+        const SketchRow cut = sketch_row(min(max(__float_as_int(nrm.w), 1), n_units), min(max(piece, 1), n_units),
+                                         full_units);
         // the k-th largest of the lanes' largest entries
         float lane_max = -INFINITY;
         for (int v0 = 0;;) {
