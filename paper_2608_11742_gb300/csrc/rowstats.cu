@@ -204,7 +204,6 @@ struct Elem<RPS_BF16> {
     typedef uint16_t Sketch;
     static constexpr uint32_t kNegInf2 = 0xff80ff80u;  // a 32-bit word of -inf sketch entries
     __device__ static __forceinline__ Sketch to_sketch(float v) { return static_cast<uint16_t>(__float_as_uint(v) >> 16); }
-    __device__ static __forceinline__ float from_sketch(Sketch s) { return __uint_as_float(static_cast<uint32_t>(s) << 16); }
     // running maximum of whole units, kept as a packed bf16 pair
     typedef uint32_t Acc;
     __device__ static __forceinline__ Acc acc_init() { return 0xff80ff80u; }  // (-inf, -inf)
@@ -240,7 +239,6 @@ struct Elem<RPS_F32> {
     typedef float Sketch;
     static constexpr uint32_t kNegInf2 = 0xff800000u;
     __device__ static __forceinline__ Sketch to_sketch(float v) { return v; }
-    __device__ static __forceinline__ float from_sketch(Sketch s) { return s; }
     typedef float Acc;
     __device__ static __forceinline__ Acc acc_init() { return -INFINITY; }
     __device__ static __forceinline__ Acc acc_add(Acc m, const uint4 &w) { return fmaxf(m, unit_max(w)); }
