@@ -48,7 +48,9 @@ class DecodeLoop:
         self.steps = torch.zeros(n_req, **i32)  # steps each request took
         self.graph = None
 
-    LAUNCHES = rps.Step.LAUNCHES + 3  # generator fill, generator advance (2 kernels), decode advance
+    # launches of the scoring graph: the step, the generator's advance (two kernels) and the
+    # decode advance (the generator's fill runs in the denoiser stub's graph)
+    LAUNCHES = rps.Step.LAUNCHES + 3
 
     def forward_stub(self, stream=None):
         synth.device_fill_blocks(self.logits, self.seed, self.mixture, self.d_step, self.block, self.L_total,
