@@ -394,10 +394,25 @@ def time_oracle(sample, k_max: int, budget_s: float):
     return done / elapsed, done, elapsed
 
 
+def host_cpu() -> dict:
+    """The host's logical CPU count and model (lscpu where present, else the platform)."""
+    import os, platform, subprocess
+    model = platform.processor() or platform.machine()
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name:"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return {"nproc": os.cpu_count(), "model": model, "machine": platform.machine()}
+
+
 def cpu_baseline(w, prm, budget_s: float):
     sample = cpu_sample(w)
     rows_s, done, elapsed = time_oracle(sample, prm.k_max, budget_s)
-    return {"value": rows_s, "unit": "rows/s", "cores": 1, "kind": "oracle",
+    return {"value": rows_s, "unit": "rows/s", "cores": 1, "kind": "oracle", "host": host_cpu(),
             "sample": f"{done} rows of the {w.name} workload ({len(sample[0])} base rows in top-k mode and "
                       f"{len(sample[1])} lookahead rows, repeated) scored by the single-threaded fp64 oracle in "
                       f"{elapsed:.1f} s ({rows_s * w.V * w.elem_bytes / 1e9:.3f} GB/s)"}
@@ -522,7 +537,7 @@ def run_reference(args):
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": None, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": describe(w), "input_dtype": w.dtype},
-           "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle",
+           "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle", "host": host_cpu(),
                             "sample": f"each step: about {per_step:.1f} s of the single-threaded fp64 oracle on a "
                                       f"64-row sample of the workload ({len(sample[0])} base rows in top-k mode, "
                                       f"{len(sample[1])} lookahead rows)"},
