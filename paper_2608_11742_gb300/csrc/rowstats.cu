@@ -1056,7 +1056,7 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
 }
 
 // ---------------------------------------------------------------- top-k launch
-// Second launch of top-k mode (k <= 32), one warp per row. Its statistics
+// Second launch of top-k mode (k <= 32), one warp per slot of the row list. Its statistics
 // launch left the row's sketch -- the maximum of every cell, a cell being one
 // lane's units of one ring chunk -- and B, ln S, 1 / S. The k-th largest of the 32
 // lanes' largest sketch entries bounds the row's k-th largest logit from below
@@ -1065,7 +1065,7 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
 // read again, and their elements at or above it enter the warp-distributed
 // sorted list (lane j = rank j, logit desc then token asc).
 constexpr int kCellCap = 256;  // candidate cells a warp buffers before reloading them
-constexpr int kSketchVecs = 24;  // 16-byte sketch loads a lane keeps in flight (a slot of <= 768 in one go)
+constexpr int kSketchVecs = 24;  // 16-byte sketch loads a lane keeps in flight (up to 768 vectors a slot in one round)
 static_assert(kSketchVecs <= 32, "one hit bit per vector");
 
 // Merges the elements at or above max(theta, current k-th entry) of the staged
