@@ -394,6 +394,15 @@ def time_oracle(sample, k_max: int, budget_s: float):
     return done / elapsed, done, elapsed
 
 
+def all_cores_entry(w, sample, k_max: int, budget_s: float) -> dict:
+    """The same oracle in one process per logical CPU at once (summed rates)."""
+    from oracle.parallel import rows_per_second_all_cores
+    rows_s, done, procs = rows_per_second_all_cores(sample, k_max, budget_s)
+    return {"value": rows_s, "unit": "rows/s", "cores": procs,
+            "sample": f"{procs} processes, each the single-threaded oracle over the same sample for about "
+                      f"{budget_s:.0f} s ({done} rows in all; {rows_s * w.V * w.elem_bytes / 1e9:.3f} GB/s)"}
+
+
 def host_cpu() -> dict:
     """The host's logical CPU count and model (lscpu where present, else the platform)."""
     import os, platform, subprocess
@@ -415,7 +424,8 @@ def cpu_baseline(w, prm, budget_s: float):
     return {"value": rows_s, "unit": "rows/s", "cores": 1, "kind": "oracle", "host": host_cpu(),
             "sample": f"{done} rows of the {w.name} workload ({len(sample[0])} base rows in top-k mode and "
                       f"{len(sample[1])} lookahead rows, repeated) scored by the single-threaded fp64 oracle in "
-                      f"{elapsed:.1f} s ({rows_s * w.V * w.elem_bytes / 1e9:.3f} GB/s)"}
+                      f"{elapsed:.1f} s ({rows_s * w.V * w.elem_bytes / 1e9:.3f} GB/s)",
+            "all_cores": all_cores_entry(w, sample, prm.k_max, min(4.0, budget_s))}
 
 
 def run_gpu(args):
@@ -540,7 +550,8 @@ def run_reference(args):
            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle", "host": host_cpu(),
                             "sample": f"each step: about {per_step:.1f} s of the single-threaded fp64 oracle on a "
                                       f"64-row sample of the workload ({len(sample[0])} base rows in top-k mode, "
-                                      f"{len(sample[1])} lookahead rows)"},
+                                      f"{len(sample[1])} lookahead rows)",
+                            "all_cores": all_cores_entry(w, sample, prm.k_max, 4.0)},
            "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
 
