@@ -689,9 +689,89 @@ def pin_propositions(o):
             assert all(la[prm.tokens_per_pivot] >= la[cs] - 1e-12 for cs in valid)
 
 
+# --------------------------------------------------------------------------
+# LM head followed by the row statistics (the oracle of a fused contraction)
+# --------------------------------------------------------------------------
+
+def _bf16_bits(x) -> np.ndarray:
+    """bf16 bits of values that bf16 holds exactly (checked)."""
+    f = np.asarray(x, dtype=np.float32)
+    bits = (f.view(np.uint32) >> 16).astype(np.uint16)
+    assert ((bits.astype(np.uint32) << 16).view(np.float32) == f).all(), "value not exact in bf16"
+    return bits
+
+
+def pin_lmhead_worked_example(o):
+    """d = 2, V = 3: h = (1, 2) and W = [[1, 0], [0, 1], [1, 1]] give z = (1, 2, 3)."""
+    from oracle.lmhead import lmhead_row_stats
+    st = lmhead_row_stats(o, _bf16_bits([[1, 2]]), _bf16_bits([[1, 0], [0, 1], [1, 1]]), 2)
+    z = np.array([1.0, 2.0, 3.0])
+    p = np.exp(z - z.max()) / np.exp(z - z.max()).sum()
+    lse = math.log(np.exp(z).sum())
+    close(st.zmax[0], 3.0, what="zmax")
+    close(st.lse[0], lse, what="lse")
+    close(st.H[0], -(p * np.log(p)).sum(), what="H")
+    close(st.pmax[0], p[2], what="pmax")
+    assert st.argmax[0] == 2
+    assert list(st.topk_idx[0, :2]) == [2, 1]
+    close(st.mu[0], p[2] + p[1], what="mu")
+    close(st.htrunc[0], -(p[2] * math.log(p[2]) + p[1] * math.log(p[1])), what="htrunc")
+
+
+def pin_lmhead_zero_hidden(o):
+    """A zero hidden state makes every logit 0: the uniform row's closed forms."""
+    from oracle.lmhead import lmhead_row_stats
+    rng = np.random.default_rng(3)
+    V, d, k = 300, 16, 10
+    w = _bf16_bits(rng.integers(-8, 9, (V, d)).astype(np.float32))
+    st = lmhead_row_stats(o, _bf16_bits(np.zeros((2, d))), w, k)
+    close(st.H, math.log(V), what="H")
+    close(st.pmax, 1.0 / V, what="pmax")
+    close(st.mu, k / V, what="mu")
+    assert (st.argmax == 0).all() and (st.topk_idx[:, :k] == np.arange(k)).all()
+
+
+def pin_lmhead_token_shift(o):
+    """Adding one vector u to every token's weights adds h.u to every logit of the
+    row: the distribution, argmax and top-k stay, zmax and lse move by h.u."""
+    from oracle.lmhead import lmhead_row_stats
+    rng = np.random.default_rng(4)
+    n, V, d, k = 4, 200, 8, 12
+    h = rng.integers(-3, 4, (n, d)).astype(np.float32)
+    w = rng.integers(-4, 5, (V, d)).astype(np.float32)
+    u = rng.integers(-2, 3, d).astype(np.float32)
+    a = lmhead_row_stats(o, _bf16_bits(h), _bf16_bits(w), k)
+    b = lmhead_row_stats(o, _bf16_bits(h), _bf16_bits(w + u), k)
+    shift = h.astype(np.float64) @ u.astype(np.float64)
+    close(b.zmax, a.zmax + shift, what="zmax")
+    close(b.lse, a.lse + shift, tol=1e-9, what="lse")
+    for name in ("H", "pmax", "mu", "htrunc"):
+        close(getattr(b, name), getattr(a, name), tol=1e-9, what=name)
+    assert (a.argmax == b.argmax).all() and (a.topk_idx == b.topk_idx).all()
+
+
+def pin_lmhead_token_permutation(o):
+    """Token v of the permuted unembedding is token perm[v] of the original: the
+    argmax and top-k tokens map back through perm (distinct logits)."""
+    from oracle.lmhead import lmhead_row_stats
+    rng = np.random.default_rng(5)
+    V, d, k = 97, 3, 7
+    w = np.zeros((V, d), np.float32)
+    w[:, 0] = rng.permutation(V)           # z_v = w[v, 0] for h = (1, 0, 0): distinct
+    w[:, 1:] = rng.integers(-5, 6, (V, d - 1))
+    h = np.array([[1, 0, 0]], np.float32)
+    perm = rng.permutation(V)
+    a = lmhead_row_stats(o, _bf16_bits(h), _bf16_bits(w), k)
+    b = lmhead_row_stats(o, _bf16_bits(h), _bf16_bits(w[perm]), k)
+    assert a.argmax[0] == int(np.argmax(w[:, 0])) and perm[b.argmax[0]] == a.argmax[0]
+    assert (perm[b.topk_idx[0, :k]] == a.topk_idx[0, :k]).all()
+    close(b.H, a.H, tol=1e-12, what="H")
+
+
 ALL_PINS = [
     pin_uniform_rows, pin_spike_rows, pin_two_level_rows, pin_rank_order, pin_library_crosscheck,
     pin_synth_rows_crosscheck, pin_invariants, pin_neg_inf_entries, pin_select_brute_force,
     pin_score_commit_brute_force, pin_score_closed_form, pin_control_flow, pin_exact_thresholds,
-    pin_propositions,
+    pin_propositions, pin_lmhead_worked_example, pin_lmhead_zero_hidden, pin_lmhead_token_shift,
+    pin_lmhead_token_permutation,
 ]

@@ -85,3 +85,33 @@ def test_mutant_is_caught(tmp_path, name, old, new):
         except AssertionError:
             return
     pytest.fail(f"mutant '{name}' passed every pin")
+
+
+# Plausible mistakes in the LM-head oracle's contraction (its statistics are the
+# row-statistics oracle's, mutated above): each must fail an LM-head pin.
+def _lm_mutants():
+    import numpy as np
+    import oracle.lmhead as lm
+    orig = lm.lmhead_logits
+    return {
+        "negated product": lambda h, w: -orig(h, w),
+        "tokens reversed": lambda h, w: orig(h, w)[:, ::-1].copy(),
+        "last weight dropped": lambda h, w: (lm.bf16_to_f64(h)[:, :-1] @ lm.bf16_to_f64(w)[:, :-1].T).astype(np.float32),
+        "product doubled": lambda h, w: 2 * orig(h, w),
+        "first row for every row": lambda h, w: np.repeat(orig(h, w)[:1], len(h), axis=0),
+    }
+
+
+@pytest.mark.parametrize("name", ["negated product", "tokens reversed", "last weight dropped", "product doubled",
+                                  "first row for every row"])
+def test_lmhead_mutant_is_caught(oracle, monkeypatch, name):
+    import oracle.lmhead as lm
+    monkeypatch.setattr(lm, "lmhead_logits", _lm_mutants()[name])
+    caught = False
+    for pin in (p for p in pins.ALL_PINS if p.__name__.startswith("pin_lmhead")):
+        try:
+            pin(oracle)
+        except Exception:
+            caught = True
+            break
+    assert caught, f"no LM-head pin catches '{name}'"
