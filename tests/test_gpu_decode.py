@@ -15,7 +15,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_harness import (assert_close, commit_np, compare_commit, compare_scores, compare_select, piv_np, scores_np,
+from gpu_harness import (MAX_EXCUSED, assert_close, commit_np, compare_commit, compare_scores, compare_select, piv_np, scores_np,
                          stats_np)
 from oracle import default as oracle_default
 from paper_2608_11742_gb300 import configs, synth
@@ -112,11 +112,12 @@ def _run_checked(prm):
             assert_close(getattr(base, name)[slots], getattr(ref, name)[slots], f"step {s} base {name}")
         assert (base.argmax[slots] == ref.argmax[slots]).all()
         piv_o = o.select_pivots(m.mask_pos, m.mask_cnt, base, prm)
-        compare_select(piv, piv_o, m.mask_cnt, B, prm.n_pivots, prm.tokens_per_pivot, set(), f"step {s} select")
+        compare_select(piv, piv_o, m.mask_cnt, B, prm.n_pivots, prm.tokens_per_pivot, {}, f"step {s} select")
         sc_o = o.score_branches(piv, br, base, z[:, 0], prm)
-        compare_scores(scores_np(st.scores), sc_o, br.pmax, prm, f"step {s} scores")
+        sc_g = scores_np(st.scores)
+        compare_scores(sc_g, sc_o, prm, f"step {s} scores")
         cm = commit_np(st.commit)
-        compare_commit(cm, o.commit(piv, sc_o, prm), sc_o, B, f"step {s} commit")
+        assert len(compare_commit(cm, o.commit(piv, sc_o, prm), sc_g, sc_o, piv, prm, f"step {s} commit")) <= MAX_EXCUSED
         winners += [int(w) for q, w in enumerate(cm["winner"]) if not m.done[q]]
         m.advance(piv, cm)
         assert np.array_equal(loop.tokens.cpu().numpy(), m.tokens), f"step {s}: response tokens"

@@ -359,16 +359,17 @@ def test_full_size_sampled(rps, name, w):
         assert (br.argmax[sl] == ref.argmax).all()
 
     # decision stages: the oracle on the GPU's statistics gives the GPU's decisions
-    from gpu_harness import compare_commit, compare_scores, compare_select, scores_np, commit_np
+    from gpu_harness import MAX_EXCUSED, compare_commit, compare_scores, compare_select, scores_np, commit_np
     piv_o = o.select_pivots(mpos, mcnt, base, prm)
-    compare_select(piv, piv_o, mcnt, w.L, prm.n_pivots, prm.tokens_per_pivot, set(), f"{name} select")
+    compare_select(piv, piv_o, mcnt, w.L, prm.n_pivots, prm.tokens_per_pivot, {}, f"{name} select")
     anchor = logits[:, 0]
     if w.dtype == "bf16":
         anchor_np = anchor.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
     else:
         anchor_np = anchor.contiguous().cpu().numpy()
     sc_o = o.score_branches(piv, br, base, anchor_np, prm)
-    compare_scores(scores_np(step.scores), sc_o, br.pmax, prm, f"{name} scores")
+    sc_g = scores_np(step.scores)
+    compare_scores(sc_g, sc_o, prm, f"{name} scores")
     cm_o = o.commit(piv, sc_o, prm)
-    compare_commit(commit_np(step.commit), cm_o, sc_o, w.L, f"{name} commit")
+    assert len(compare_commit(commit_np(step.commit), cm_o, sc_g, sc_o, piv, prm, f"{name} commit")) <= MAX_EXCUSED
     assert (piv["state"] == 0).any(), "the exercise setting must reach the lookahead search"

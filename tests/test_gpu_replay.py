@@ -13,7 +13,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_harness import (GpuStep, assert_close, commit_np, compare_commit, compare_scores, compare_select, piv_np,
+from gpu_harness import (MAX_EXCUSED, GpuStep, assert_close, commit_np, compare_commit, compare_scores, compare_select, piv_np,
                          scores_np, stats_np)
 from oracle import default as oracle_default
 from paper_2608_11742_gb300 import configs, rps, synth
@@ -76,13 +76,14 @@ def test_long_replay_full_size():
 
         # the decisions are the oracle's on the GPU's statistics
         piv_o = o.select_pivots(mpos, mcnt, base, prm)
-        compare_select(piv, piv_o, mcnt, w.L, prm.n_pivots, prm.tokens_per_pivot, set(), f"step {s} select")
+        compare_select(piv, piv_o, mcnt, w.L, prm.n_pivots, prm.tokens_per_pivot, {}, f"step {s} select")
         anchor = logits[:, 0].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
         sc_o = o.score_branches(piv, br, base, anchor, prm)
-        compare_scores(scores_np(step.scores), sc_o, br.pmax, prm, f"step {s} scores")
+        sc_g = scores_np(step.scores)
+        compare_scores(sc_g, sc_o, prm, f"step {s} scores")
         cm_o = o.commit(piv, sc_o, prm)
         cm = commit_np(step.commit)
-        compare_commit(cm, cm_o, sc_o, w.L, f"step {s} commit")
+        assert len(compare_commit(cm, cm_o, sc_g, sc_o, piv, prm, f"step {s} commit")) <= MAX_EXCUSED
         winners.append(int(cm["winner"][0]))
         st.advance(cm["winner"], cm["mask_pos"], cm["mask_cnt"])
     assert len(winners) == STEPS, "512 positions outlast 64 steps"
