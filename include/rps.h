@@ -69,7 +69,10 @@ typedef enum {
 #define RPS_DEVERR_MASK 0x4u       /* mask count above capacity or position out of range */
 #define RPS_DEVERR_TOKEN 0x8u      /* candidate token outside the vocabulary */
 #define RPS_DEVERR_TIMEOUT 0x10u   /* a bounded wait for an asynchronous copy gave up; the call's
-                                      outputs are incomplete and its workspace must be re-zeroed */
+                                      outputs are incomplete and its workspace is marked unhealthy */
+#define RPS_DEVERR_WORKSPACE 0x20u /* the workspace was marked unhealthy by an earlier call that gave
+                                      up (or holds a stale ticket): the call wrote no statistics;
+                                      rps_workspace_init makes the workspace usable again */
 
 typedef enum { RPS_F32 = 0, RPS_BF16 = 1 } rps_dtype;
 
@@ -207,7 +210,11 @@ size_t rps_workspace_bytes(int64_t max_rows, int64_t vocab, int32_t dtype, int32
 
 /* Zero a workspace (asynchronously on `stream`). A workspace must be zeroed
  * once before its first use; every completed rps_score_step leaves it ready
- * for the next call. One workspace must not serve two calls that can overlap. */
+ * for the next call. One workspace must not serve two calls that can overlap.
+ * Its first 256 bytes hold a health word: a call whose kernel gives up on a
+ * bounded wait (RPS_DEVERR_TIMEOUT) leaves row tickets unfinished and marks
+ * the word, and every later call on that workspace writes no statistics and
+ * reports RPS_DEVERR_WORKSPACE until the workspace is zeroed again. */
 rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream);
 
 /*
@@ -362,6 +369,10 @@ rps_status rps_gather_rows(const rps_logits *src, const rps_row_list *rows, cons
  *     the part of the array it uses with cudaMemsetAsync on `stream`.
  *   - The first call on each device looks up the array's device address while
  *     that device is current; make that first call before any stream capture.
+ *     The address is kept for the life of the process: after cudaDeviceReset
+ *     (or anything else that destroys the device's primary context) it no
+ *     longer names the array, so do not call this function on that device
+ *     again in the same process.
  *   - All calls on a device share the one array: calls that can overlap on the
  *     GPU (different streams without ordering between them) race and corrupt each
  *     other's results. Order them on one stream or serialise them.
@@ -373,6 +384,14 @@ rps_status rps_score_step_noalloc(const rps_logits *logits, const rps_row_list *
  * Returns RPS_OK or RPS_ERR_DEVICE (with the RPS_DEVERR_* bits in *detail when
  * detail != NULL), or RPS_ERR_CUDA if the synchronisation itself failed. */
 rps_status rps_poll_device_status(rps_stream_t stream, uint32_t *detail);
+
+/* Testing hook, no counterpart in the paper: sets the limit of the
+ * row-statistics kernels' wait for each asynchronous row copy (200 ms by
+ * default, restored by UINT64_MAX; 0 makes every such wait give up at once,
+ * so that a test can see a timeout reported). It applies to calls enqueued
+ * after it, process-wide. The copies already issued are still waited for
+ * (200 ms each) before a warp that gave up stops. Returns the previous limit. */
+uint64_t rps_debug_set_ring_wait_ns(uint64_t ns);
 
 /* Static description of a status code. */
 const char *rps_status_string(rps_status status);

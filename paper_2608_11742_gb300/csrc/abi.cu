@@ -3,6 +3,7 @@
 #include <cmath>
 #include <algorithm>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include "rps_internal.cuh"
@@ -25,6 +26,11 @@ struct DeviceInfo {
 
 std::mutex g_mutex;
 DeviceInfo g_devices[kMaxDevices];
+
+// Limit of the row-statistics kernels' wait for each ring chunk (see
+// rps_debug_set_ring_wait_ns).
+constexpr uint64_t kRingWaitNs = 200ull * 1000 * 1000;
+std::atomic<uint64_t> g_ring_wait_ns{kRingWaitNs};
 
 size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
@@ -82,19 +88,21 @@ rps_status check_logits(const rps_logits *l) {
 }
 
 struct WorkspaceLayout {
-    size_t ticket, part, sketch, norm, piece, total;
+    size_t health, ticket, part, sketch, norm, piece, total;
 };
 
-// Tickets, partial records, and in top-k mode the sketch (one element-sized
-// entry per cell: one lane's units of one 2 KB ring chunk), each row's B, ln S,
-// 1 / S and first piece length, and the launch's piece length.
+// The health word (its own 256-byte line), tickets, partial records, and in
+// top-k mode the sketch (one element-sized entry per cell: one lane's units of
+// one 2 KB ring chunk), each row's B, ln S, 1 / S and first piece length, and
+// the launch's piece length.
 WorkspaceLayout layout(int64_t max_rows, int64_t vocab, int32_t dtype, int32_t k) {
     WorkspaceLayout w;
     const size_t rows = static_cast<size_t>(max_rows);
     const size_t esize = dtype == RPS_BF16 ? 2 : 4;
     const size_t units = (static_cast<size_t>(vocab) * esize + 15) / 16;
-    w.ticket = 0;
-    w.part = align_up(rows * sizeof(uint32_t));
+    w.health = 0;
+    w.ticket = kAlign;
+    w.part = w.ticket + align_up(rows * sizeof(uint32_t));
     w.sketch = w.part + align_up(rows * kMaxPartials * sizeof(Partial));
     w.norm = w.sketch + (k > 0 ? align_up(rows * static_cast<size_t>(sketch_entries(units)) * esize) : 0);
     w.piece = w.norm + (k > 0 ? align_up(rows * sizeof(float4)) : 0);
@@ -133,25 +141,37 @@ rps_status rps_workspace_init(void *d_ws, size_t ws_bytes, rps_stream_t stream) 
 namespace rps {
 namespace {
 
-// Checks the arguments of a row-statistics launch and fills its kernel
-// arguments and grid.
-rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
-                             const rps_row_stats *out, void *d_ws, size_t ws_bytes, RowStatsArgs *ap,
-                             int *grid_out, int *topk_grid_out) {
+}  // namespace
+
+rps_status check_row_stats_args(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                                const rps_row_stats *out, int32_t *k_out) {
     rps_status st = check_logits(logits);
     if (st != RPS_OK) return st;
     if (!rows || (!rows->rows && !rows->mask_pos) || rows->n_seg < 1 || rows->cap < 1) return RPS_ERR_INVALID_ARG;
     if (rows->n_seg > RPS_MAX_SEGMENTS) return RPS_ERR_UNSUPPORTED;
     if (static_cast<int64_t>(rows->n_seg) * rows->cap > INT32_MAX / 3) return RPS_ERR_INVALID_ARG;
     if (!out || !out->zmax || !out->lse || !out->H || !out->pmax || !out->argmax) return RPS_ERR_INVALID_ARG;
-    const bool topk = out->topk_idx != nullptr;
     int32_t k = 0;
-    if (topk) {
+    if (out->topk_idx) {
         if ((st = check_params(prm, false)) != RPS_OK) return st;
         if (!out->topk_logit || !out->mu || !out->htrunc) return RPS_ERR_INVALID_ARG;
         if (prm->k_max > logits->vocab) return RPS_ERR_INVALID_ARG;
         k = prm->k_max;
     }
+    *k_out = k;
+    return RPS_OK;
+}
+
+namespace {
+
+// Checks the arguments of a row-statistics launch and fills its kernel
+// arguments and grid.
+rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                             const rps_row_stats *out, void *d_ws, size_t ws_bytes, RowStatsArgs *ap,
+                             int *grid_out, int *topk_grid_out) {
+    int32_t k = 0;
+    rps_status st = check_row_stats_args(logits, rows, prm, out, &k);
+    if (st != RPS_OK) return st;
     const int64_t max_rows = static_cast<int64_t>(rows->n_seg) * rows->cap;
     const WorkspaceLayout w = layout(max_rows, logits->vocab, logits->dtype, k);
     if (!d_ws || ws_bytes < w.total || reinterpret_cast<uintptr_t>(d_ws) % 16 != 0) return RPS_ERR_INVALID_ARG;
@@ -189,6 +209,8 @@ rps_status prepare_row_stats(const rps_logits *logits, const rps_row_list *rows,
     a.topk_logit = out->topk_logit;
     char *ws = static_cast<char *>(d_ws);
     a.ticket = reinterpret_cast<uint32_t *>(ws + w.ticket);
+    a.health = reinterpret_cast<uint32_t *>(ws + w.health);
+    a.ring_wait_ns = g_ring_wait_ns.load(std::memory_order_relaxed);
     a.part = reinterpret_cast<Partial *>(ws + w.part);
     a.sketch = k > 0 ? static_cast<void *>(ws + w.sketch) : nullptr;
     a.norm = k > 0 ? reinterpret_cast<float4 *>(ws + w.norm) : nullptr;
@@ -477,6 +499,10 @@ const char *rps_status_string(rps_status status) {
     return "unknown rps_status";
 }
 
-int32_t rps_version(void) { return 200; }
+int32_t rps_version(void) { return 300; }
+
+uint64_t rps_debug_set_ring_wait_ns(uint64_t ns) {
+    return g_ring_wait_ns.exchange(ns == UINT64_MAX ? kRingWaitNs : ns);
+}
 
 }  // extern "C"

@@ -59,6 +59,7 @@ constexpr float kSlack = 8.0f;          // nats the reference may trail the maxi
 constexpr int kChunkUnits = 32 * kBatch;  // 16-byte units per ring buffer (2 KB)
 constexpr int kCandBatch = 32;  // top-k candidates merged at a time
 constexpr uint64_t kWaitLimitNs = 200ull * 1000 * 1000;  // a bulk copy normally lands within microseconds
+constexpr uint32_t kUnhealthy = 1u;  // health word of a workspace a launch gave up on
 
 // ---------------------------------------------------------------- PTX helpers
 __device__ __forceinline__ float ex2(float x) {
@@ -163,11 +164,12 @@ __device__ __forceinline__ uint64_t global_ns() {
     return t;
 }
 
-// Waits for phase `parity` of `bar`, giving up after kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+// Waits for phase `parity` of `bar`, giving up after limit_ns (at once when 0).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity, uint64_t limit_ns = kWaitLimitNs) {
+    if (limit_ns == 0) return false;
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t start = global_ns();
-    while (global_ns() - start < kWaitLimitNs)
+    while (global_ns() - start < limit_ns)
         if (mbar_try_wait(bar, parity)) return true;
     return false;
 }
@@ -864,7 +866,15 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
     uint4 *ring = dyn + wib * (kRing * kChunkUnits);
     uint64_t *bar = bars[wib];
 
+    // (loaded here, tested after the row count, so that the two loads overlap)
+    const uint32_t health = __ldcg(a.health);
     const int64_t total_rows = count_rows<kStatThreads>(a, seg_start, warp_total, lane, wib);
+    // A workspace an earlier launch gave up on holds tickets of rows it never
+    // finished: merging on them would write wrong rows, so nothing is written.
+    if (health != 0) {
+        if (threadIdx.x == 0) flag_error(a.err, RPS_DEVERR_WORKSPACE);
+        return;
+    }
 
     const int64_t nv = a.units_per_row;
     const int64_t total = total_rows * nv;
@@ -916,17 +926,21 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
     issued = __shfl_sync(kFull, issued, 0);
     int acquired = 0, released = 0;
 
-    // Waits for the next ring chunk; false when the copy never lands (then this
-    // warp has flagged the error and drained its other copies: it must stop).
+    // Waits for the next ring chunk; false when it does not land within the
+    // limit. The warp then flags the error, marks the workspace unhealthy (its
+    // rows' tickets stay incomplete), waits -- bounded -- for every copy it
+    // issued, the one that timed out included, so that none still writes into
+    // its ring, and must stop.
     auto acquire = [&](int &st) -> bool {
         st = acquired % kRing;
-        if (mbar_wait_bounded(bar + st, (acquired / kRing) & 1)) {
+        if (mbar_wait_bounded(bar + st, (acquired / kRing) & 1, a.ring_wait_ns)) {
             ++acquired;
             return true;
         }
         if (lane == 0) {
             flag_error(a.err, RPS_DEVERR_TIMEOUT);
-            for (int c = acquired + 1; c < issued; ++c) mbar_wait_bounded(bar + (c % kRing), (c / kRing) & 1);
+            atomicExch(a.health, kUnhealthy);
+            for (int c = acquired; c < issued; ++c) mbar_wait_bounded(bar + (c % kRing), (c / kRing) & 1);
         }
         __syncwarp();
         return false;
@@ -1029,7 +1043,12 @@ __global__ void __launch_bounds__(kStatThreads, kStatBlocksPerSm) row_stats_kern
         __threadfence();
         __syncwarp();
         unsigned prior = 0;
-        if (lane == 0) prior = atomicAdd(a.ticket + slot, 1u);
+        if (lane == 0) {
+            prior = atomicAdd(a.ticket + slot, 1u);
+            // a ticket at or past the piece count was left by an unfinished
+            // launch or was never zeroed
+            if (prior >= static_cast<unsigned>(count)) flag_error(a.err, RPS_DEVERR_WORKSPACE);
+        }
         prior = __shfl_sync(kFull, prior, 0);
         if (prior != static_cast<unsigned>(count - 1)) continue;
 
@@ -1218,9 +1237,14 @@ __global__ void __launch_bounds__(kTopkWarps * 32, kTopkMinBlocks) topk_rows_ker
         const float zmax = __ldcg(a.zmax + slot);
         const float4 nrm = __ldcg(a.norm + slot);
         const int piece = __ldcg(a.sketch_piece);
+        const uint32_t health = __ldcg(a.health);
         // Pass 1: the largest entry of each of this lane's vectors v0 + 32 q + lane.
         float vm[kSketchVecs];
         vector_maxima<DT>(vm, sk, 0, n_vec, lane);
+        if (health != 0) {  // the statistics launch gave up, or found the workspace unhealthy
+            if (lane == 0) flag_error(a.err, RPS_DEVERR_WORKSPACE);
+            break;
+        }
         if (zmax != zmax) {  // the statistics launch found no finite row
             if (lane == 0) {
                 a.argmax[slot] = -1;

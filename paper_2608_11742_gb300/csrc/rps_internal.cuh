@@ -77,6 +77,8 @@ struct RowStatsArgs {
     float4 *norm;         // [slots] B, ln S, 1 / S of each row's base-2 softmax and its sketch's len0 (top-k mode)
     int32_t *sketch_piece;  // [1] units per piece of the sketch layout (top-k mode)
     uint32_t *ticket;     // [slots]
+    uint32_t *health;     // workspace health word: 0, or non-zero once a launch on this workspace gave up
+    uint64_t ring_wait_ns;  // limit of a warp's wait for its next ring chunk (0: give up at once)
     // decomposition: the rows' 16-byte units are split evenly over `warps` warps
     int64_t units_per_row;
     int32_t warps;
@@ -133,6 +135,12 @@ cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStr
 
 // The calling device's sticky error word (nullptr if the device cannot be queried).
 uint32_t *device_error_word();
+
+// The host-side argument rules of rps_score_step (everything but the
+// workspace), checked before anything is enqueued; *k_out is the top-k size
+// (0 in statistics-only mode). Shared by every row-statistics entry point.
+rps_status check_row_stats_args(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
+                                const rps_row_stats *out, int32_t *k_out);
 
 // ---------------------------------------------------------------- launches
 // Every kernel of the library is launched with programmatic stream

@@ -32,33 +32,15 @@ rps_status scratch_for_current_device(void **out) {
     return RPS_OK;
 }
 
-// Same argument rules as rps_score_step, checked before anything is enqueued.
-bool arguments_ok(const rps_logits *l, const rps_row_list *rows, const rps_params *prm, const rps_row_stats *out) {
-    if (!l || !l->data || (l->dtype != RPS_F32 && l->dtype != RPS_BF16)) return false;
-    if (l->vocab < 1 || l->vocab > INT32_MAX || l->n_req < 1 || l->n_branch < 1 || l->n_pos < 1) return false;
-    if (l->req_stride < 0 || l->branch_stride < 0 || l->pos_stride < 0) return false;
-    const int64_t esize = l->dtype == RPS_BF16 ? 2 : 4;
-    if (reinterpret_cast<uintptr_t>(l->data) % 16 || (l->req_stride * esize) % 16 || (l->branch_stride * esize) % 16 ||
-        (l->pos_stride * esize) % 16)
-        return false;
-    if (!rows || (!rows->rows && !rows->mask_pos) || rows->n_seg < 1 || rows->cap < 1) return false;
-    if (static_cast<int64_t>(rows->n_seg) * rows->cap > INT32_MAX / 3) return false;
-    if (!out || !out->zmax || !out->lse || !out->H || !out->pmax || !out->argmax) return false;
-    if (out->topk_idx && (!prm || prm->k_max < 1 || prm->k_max > l->vocab || !out->topk_logit || !out->mu ||
-                          !out->htrunc))
-        return false;
-    return true;
-}
-
 }  // namespace
 
 extern "C" rps_status rps_score_step_noalloc(const rps_logits *logits, const rps_row_list *rows,
                                              const rps_params *prm, const rps_row_stats *out,
                                              rps_stream_t stream) {
-    if (out && out->topk_idx && prm && prm->k_max > RPS_MAX_K) return RPS_ERR_UNSUPPORTED;
-    if (rows && rows->n_seg > RPS_MAX_SEGMENTS) return RPS_ERR_UNSUPPORTED;
-    if (!arguments_ok(logits, rows, prm, out)) return RPS_ERR_INVALID_ARG;
-    const int32_t k = out->topk_idx ? prm->k_max : 0;
+    // the argument rules of rps_score_step, checked before anything is enqueued
+    int32_t k = 0;
+    const rps_status arg = rps::check_row_stats_args(logits, rows, prm, out, &k);
+    if (arg != RPS_OK) return arg;
     const size_t need =
         rps_workspace_bytes(static_cast<int64_t>(rows->n_seg) * rows->cap, logits->vocab, logits->dtype, k);
     if (need == 0) return RPS_ERR_INVALID_ARG;
@@ -68,8 +50,8 @@ extern "C" rps_status rps_score_step_noalloc(const rps_logits *logits, const rps
     const rps_status st = scratch_for_current_device(&scratch);
     if (st != RPS_OK) return st;
     // The array keeps whatever the previous call left; the per-row completion
-    // tickets must start at zero, so the part of the array this call uses is
-    // cleared on the call's stream (a memset, no allocation).
+    // tickets and the health word must start at zero, so the part of the array
+    // this call uses is cleared on the call's stream (a memset, no allocation).
     if (cudaMemsetAsync(scratch, 0, need, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return RPS_ERR_CUDA;
     return rps_score_step(logits, rows, prm, out, scratch, RPS_STATIC_SCRATCH_BYTES, stream);
 }

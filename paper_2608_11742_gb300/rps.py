@@ -32,6 +32,7 @@ RPS_F32, RPS_BF16 = 0, 1
 STATE_SEARCH, STATE_DONE, STATE_NO_FEASIBLE, STATE_NO_CANDIDATES = 0, 1, 2, 3
 WIN_ANCHOR, WIN_SKIP, WIN_DONE = -1, -2, -3
 DEVERR_ROW_INDEX, DEVERR_NONFINITE, DEVERR_MASK, DEVERR_TOKEN = 0x1, 0x2, 0x4, 0x8
+DEVERR_TIMEOUT, DEVERR_WORKSPACE = 0x10, 0x20
 
 _p = C.c_void_p
 
@@ -114,6 +115,8 @@ _lib.rps_status_string.restype = C.c_char_p
 _lib.rps_status_string.argtypes = [C.c_int]
 _lib.rps_version.restype = C.c_int32
 _lib.rps_version.argtypes = []
+_lib.rps_debug_set_ring_wait_ns.restype = C.c_uint64
+_lib.rps_debug_set_ring_wait_ns.argtypes = [C.c_uint64]
 
 
 class RPSError(RuntimeError):
@@ -254,6 +257,12 @@ class CommitBuf:
 # --------------------------------------------------------------------------- ABI calls
 def rps_version() -> int:
     return _lib.rps_version()
+
+
+def rps_debug_set_ring_wait_ns(ns: int) -> int:
+    """Testing hook: the row-statistics kernels' limit on each ring-copy wait
+    (0 gives up at once; ``2**64 - 1`` restores the default). Returns the previous limit."""
+    return _lib.rps_debug_set_ring_wait_ns(ns)
 
 
 def rps_status_string(status: int) -> str:
