@@ -5,8 +5,14 @@ rps_score_branches / rps_commit) on GB300.
 A step is one pass of the whole path over one decoding step's synthetic logits:
 row statistics of the masked base rows (top-k mode), standard commit and pivot
 selection, row statistics of the lookahead rows, benefit scores and the commit
-decision. The headline workload is one generation step: 256 masked positions,
-vocab 126,464, bf16 logits, 1 base + 8 lookahead branches (4 pivots x top-2).
+decision. The headline workload is the largest one that fits one GPU, the
+batched serving step: 8 requests x 256 positions, vocab 151,936, bf16 logits,
+1 base + 16 lookahead branches (8 pivots x top-2), ragged masked counts
+U{16..256} with NaN-padded unmasked rows. Every other workload (the generation
+step at 100 / 50 / 10 % masked, the long generation's first step and its whole
+64-step replay, the KV-cache block step and the tiny fp32 step) gets a record of
+its own under `per_workload`, each with the roofline of its lookahead
+row-statistics launch and its whole-step fraction of the HBM peak.
 
 Timing: the launches of a step are captured in one CUDA graph; each timed
 replay is preceded by an L2 flush (a 256 MB buffer is written, then read back,
@@ -44,8 +50,9 @@ ROOT = Path(__file__).resolve().parent
 sys.path.insert(0, str(ROOT))
 
 METRIC = "lookahead-scoring logit rows/s and achieved HBM GB/s (fraction of GB300 peak)"
-HEADLINE = "step"
-OTHERS = ("step-50", "step-10", "long", "block", "serve")
+HEADLINE = "serve"
+OTHERS = ("step", "step-50", "step-10", "long", "block", "tiny")
+REPLAY_STEPS = 64
 FLUSH_BYTES = 256 << 20
 FALLBACK_HBM_GBS = 6800.0
 KERNEL_SOURCES = ("paper_2608_11742_gb300/csrc/rowstats.cu", "paper_2608_11742_gb300/csrc/rps_internal.cuh")
@@ -335,6 +342,71 @@ class Workload:
         return ms, h2d, d2h, ms_full, h2d_full
 
 
+def workload_record(x, step_ms, peak: float, peak_kind: str) -> dict:
+    """Step time, whole-step HBM fraction and the roofline of the dominant
+    (lookahead row-statistics) launch of one timed workload."""
+    ts = statistics.mean(step_ms)
+    kernel_us = {k: statistics.mean(v) * 1e3 for k, v in x.kernel_ms.items() if v}
+    la_ms = kernel_us["lookahead_rows"] / 1e3
+    base_ms = kernel_us["base_rows_topk"] / 1e3
+    la_gbs = x.branch_bytes() / (la_ms / 1e3) / 1e9
+    base_bytes = x.base_rows * x.w.V * x.w.elem_bytes
+    return {"workload": describe(x.w), "rows_per_step": x.rows(), "base_rows": x.base_rows,
+            "lookahead_rows": x.branch_rows, "bytes_per_step": x.bytes(),
+            "step_us": ts * 1e3, "p50_step_us": statistics.median(step_ms) * 1e3,
+            "p90_step_us": sorted(step_ms)[int(0.9 * (len(step_ms) - 1))] * 1e3,
+            "rows_per_s": x.rows() / (ts / 1e3), "gbs": x.bytes() / (ts / 1e3) / 1e9,
+            "frac": x.bytes() / (ts / 1e3) / 1e9 / peak,
+            "kernel_us": kernel_us,
+            "roofline": {"bound": "hbm", "kernel": "row statistics of the lookahead rows (statistics-only mode)",
+                         "algorithmic_bytes_per_launch": x.branch_bytes(), "launch_ms": la_ms, "achieved": la_gbs,
+                         "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": la_gbs / peak},
+            "base_launches": {"kernel": "row statistics of the masked base rows with the top-k sketch, then the "
+                                        "top-k search (two launches)",
+                              "algorithmic_bytes_per_launch": base_bytes, "launch_ms": base_ms,
+                              "achieved": base_bytes / (base_ms / 1e3) / 1e9,
+                              "frac": base_bytes / (base_ms / 1e3) / 1e9 / peak}}
+
+
+def long_replay(configs, device, flush, peak: float) -> dict:
+    """The long workload's whole 64-step replay (1 request x 512 positions, vocab
+    126,464, 1 base + 16 branches): each step's logits are written by the seeded
+    generator and L2 is flushed outside the timed region; the step then scores
+    them, and the decision moves the generator (a committed branch becomes the
+    next base, a skip draws fresh noise) and the mask (committed positions leave
+    it) for the next step, all on the device."""
+    import torch
+    from paper_2608_11742_gb300.decode import DecodeLoop
+    w = configs.LONG
+    prm = w.params(configs.EXERCISE)
+    loop = DecodeLoop(w.n_req, w.L, w.L, w.V, prm, w.seed, w.mixture, device)
+    stream = torch.cuda.Stream(device)
+    base_n, branch_n = [], []
+
+    def between():
+        flush()
+        base_n.append(loop.mask_cnt.sum())
+
+    def after():
+        branch_n.append(loop.step.piv.n_branch_rows.sum())
+
+    steps, score_ms, _ = loop.run_split(stream, max_steps=REPLAY_STEPS, between=between, after=after)
+    base = [int(v) for v in torch.stack(base_n[:steps]).cpu()]
+    branch = [int(v) for v in torch.stack(branch_n[:steps]).cpu()]
+    rows = sum(base) + sum(branch)
+    t = sum(score_ms) / 1e3
+    gbs = rows * w.V * w.elem_bytes / t / 1e9
+    del loop
+    return {"workload": describe(w) + f", replayed for {steps} decode steps on the device",
+            "steps": steps, "rows": rows, "base_rows_first_last": [base[0], base[-1]],
+            "lookahead_rows_first_last": [branch[0], branch[-1]],
+            "rows_per_s": rows / t, "gbs": gbs, "frac": gbs / peak,
+            "mean_step_us": statistics.mean(score_ms) * 1e3, "p50_step_us": statistics.median(score_ms) * 1e3,
+            "timing": "CUDA events around each step's scoring graph (the five launches of the step); the "
+                      "generator's write of the step's 2.2 GB of logits, an L2 flush and the decision's "
+                      "advance of the generator and the mask run outside the timed region"}
+
+
 def decode_run(configs, device):
     """A whole response decoded on the device (Algorithm 1): the block workload's
     64 requests x 32-position blocks extended to 256 positions. The denoiser
@@ -359,8 +431,9 @@ def decode_run(configs, device):
             "total_ms_with_stub": total_ms,
             "launches_per_step": DecodeLoop.LAUNCHES,
             "timing": "CUDA events around the graph of the scoring step (row statistics, selection, lookahead "
-                      "rows, scores and commit, decode advance), replayed after the stub's graph wrote the step's "
-                      "4.66 GB of logits (larger than L2)"}
+                      "rows, scores and commit), replayed after the stub's graph wrote the step's 4.66 GB of "
+                      "logits (larger than L2); the generator's and the decode state's advance (three launches) "
+                      "replay after it, outside the timed region"}
 
 
 def cpu_sample(w, n_take: int = 64):
@@ -447,15 +520,14 @@ def run_gpu(args):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
-        step_ms, k1_ms = wl.time(args.steps, args.warmup, flush)
+        step_ms, _ = wl.time(args.steps, args.warmup, flush)
     clocks = clk.summary()
     t_step = max_over_ranks(statistics.mean(step_ms))
     rows = wl.rows()
     value = whole_job_rate(rows, world, t_step)
-    k1 = statistics.mean(k1_ms)
-    achieved = wl.branch_bytes() / (k1 / 1e3) / 1e9
     traffic = recorded_traffic(args.workload)
 
+    rec = workload_record(wl, step_ms, peak, peak_kind)
     out = {
         "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t_step, "higher_is_better": True, "scaling": "weak",
@@ -470,34 +542,28 @@ def run_gpu(args):
                    "parallelism": f"{world} independent replica(s), no collective"},
         "achieved_gbs": wl.bytes() / (t_step / 1e3) / 1e9,
         "frac_of_hbm_peak": wl.bytes() / (t_step / 1e3) / 1e9 / peak,
-        "roofline": {"bound": "hbm", "kernel": "row statistics of the lookahead rows (statistics-only mode)",
-                     "achieved": achieved, "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic,
-                     "algorithmic_bytes_per_launch": wl.branch_bytes(), "launch_ms": k1},
+        "roofline": dict(rec["roofline"], traffic=traffic),
         "clocks": clocks,
         "gpu_launches": rps.Step.LAUNCHES * args.steps,
-        "kernel_us": {k: statistics.mean(v) * 1e3 for k, v in wl.kernel_ms.items() if v},
+        "kernel_us": rec["kernel_us"],
+        "p50_step_us": rec["p50_step_us"],
+        "base_launches": rec["base_launches"],
     }
     del wl
     torch.cuda.empty_cache()
 
     if not args.skip_others:
-        others = {}
+        per = {}
         for name in OTHERS:
             wo = configs.ALL[name]
             x = Workload(wo, wo.params(configs.EXERCISE), device)
-            sm, km = x.time(max(5, args.steps // 2), 3, flush)
-            ts = statistics.mean(sm)
-            kk = statistics.mean(km)
-            others[name] = {"rows_per_step": x.rows(), "step_us": ts * 1e3, "p50_step_us": statistics.median(sm) * 1e3,
-                            "kernel_us": {k: statistics.mean(v) * 1e3 for k, v in x.kernel_ms.items() if v},
-                            "p90_step_us": sorted(sm)[int(0.9 * (len(sm) - 1))] * 1e3,
-                            "rows_per_s": x.rows() / (ts / 1e3), "gbs": x.bytes() / (ts / 1e3) / 1e9,
-                            "frac": x.bytes() / (ts / 1e3) / 1e9 / peak,
-                            "lookahead_kernel_gbs": x.branch_bytes() / (kk / 1e3) / 1e9}
+            sm, _ = x.time(max(5, args.steps // 2), 3, flush)
+            per[name] = workload_record(x, sm, peak, peak_kind)
             del x
             torch.cuda.empty_cache()
-        out["other_workloads"] = others
+        per["long-replay"] = long_replay(configs, device, flush, peak)
+        torch.cuda.empty_cache()
+        out["per_workload"] = per
 
     if not args.skip_decode:
         out["decode"] = decode_run(configs, device)

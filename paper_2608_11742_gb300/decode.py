@@ -48,7 +48,7 @@ class DecodeLoop:
         self.steps = torch.zeros(n_req, **i32)  # steps each request took
         self.graph = None
 
-    # launches of the scoring graph: the step, the generator's advance (two kernels) and the
+    # launches of one step: the scoring step, the generator's advance (two kernels) and the
     # decode advance (the generator's fill runs in the denoiser stub's graph)
     LAUNCHES = rps.Step.LAUNCHES + 3
 
@@ -56,13 +56,19 @@ class DecodeLoop:
         synth.device_fill_blocks(self.logits, self.seed, self.mixture, self.d_step, self.block, self.L_total,
                                  self.scale, self.epoch, stream)
 
-    def score_and_advance(self, stream=None):
+    def score(self, stream=None):
+        self.step.run(self.logits, self.mask_pos, self.mask_cnt, stream)
+
+    def advance(self, stream=None):
         st = self.step
-        st.run(self.logits, self.mask_pos, self.mask_cnt, stream)
         synth.device_advance(st.commit.winner, self.B, self.L_total, self.block, self.d_step, self.scale,
                              self.epoch, self.seed, stream)
         rps.rps_decode_advance(st.piv, st.commit, self.n_req, self.B, self.L_total, self.tokens, self.block,
                                self.mask_pos, self.mask_cnt, self.done, self.steps, stream)
+
+    def score_and_advance(self, stream=None):
+        self.score(stream)
+        self.advance(stream)
 
     def step_once(self, stream=None):
         self.forward_stub(stream)
@@ -91,41 +97,53 @@ class DecodeLoop:
         self.d_step.zero_()
         self.steps.zero_()
 
-    def run_split(self, stream, check_every: int = 8):
-        """Decode to the end with the forward stub and the scoring step captured as
-        two graphs, timing each scoring replay with CUDA events on ``stream``.
+    def run_split(self, stream, check_every: int = 8, max_steps: int | None = None, between=None, after=None):
+        """Decode to the end (or for max_steps steps) with the forward stub, the
+        scoring step and the state's advance captured as three graphs, timing each
+        scoring replay (the five launches of ``rps.Step.run``) with CUDA events on
+        ``stream``. ``between`` and ``after`` (optional) run on ``stream`` outside
+        the timed region, after each stub replay and after each scoring replay (an
+        L2 flush, a row count).
         Returns (steps, per-step scoring ms, total ms)."""
         with torch.cuda.stream(stream):
             self.step_once(stream)
         stream.synchronize()
         self.reset()
-        g_fwd, g_score = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        g_fwd, g_score, g_adv = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_fwd, stream=stream):
             self.forward_stub(stream)
         with torch.cuda.graph(g_score, stream=stream):
-            self.score_and_advance(stream)
+            self.score(stream)
+        with torch.cuda.graph(g_adv, stream=stream):
+            self.advance(stream)
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         ev = []
         with torch.cuda.stream(stream):
             t0.record(stream)
         steps = 0
-        while steps < self.L_total:
-            for _ in range(check_every):
+        limit = self.L_total if max_steps is None else min(max_steps, self.L_total)
+        while steps < limit:
+            for _ in range(min(check_every, limit - steps)):
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 with torch.cuda.stream(stream):
                     g_fwd.replay()
+                    if between is not None:
+                        between()
                     e0.record(stream)
                     g_score.replay()
                     e1.record(stream)
+                    if after is not None:
+                        after()
+                    g_adv.replay()
                 ev.append((e0, e1))
-            steps += check_every
+            steps += min(check_every, limit - steps)
             stream.synchronize()
             if bool(self.done.all()):
                 break
         with torch.cuda.stream(stream):
             t1.record(stream)
         stream.synchronize()
-        taken = int(self.steps.max().item())
+        taken = min(int(self.steps.max().item()), steps) if bool(self.done.all()) else steps
         score_ms = [a.elapsed_time(b) for a, b in ev[:taken]]
         return taken, score_ms, t0.elapsed_time(t1)
 
