@@ -1,7 +1,6 @@
 // decide_device.cuh -- the per-request decision steps of one RPS step as
-// block-level device functions, shared by the decision kernels (decide.cu) and
-// the row-statistics kernel that runs them for the requests it completes
-// (rowstats.cu).
+// block-level device functions; the decision kernels of decide.cu run them,
+// one block per request.
 //
 //   select_request        standard commit (Eq. 2 with the fallback of
 //                         Algorithm 1), M' = M \ S, pivots (Eq. 3), candidate
