@@ -380,6 +380,49 @@ rps_status rps_gather_rows(const rps_logits *src, const rps_row_list *rows, cons
 rps_status rps_score_step_noalloc(const rps_logits *logits, const rps_row_list *rows, const rps_params *prm,
                                   const rps_row_stats *out, rps_stream_t stream);
 
+/*
+ * LM head with the row statistics in its epilogue (Sec. 2 notation: p_i is
+ * the softmax of the denoiser's logits for position i; Eq. 1; Eq. 3). For each
+ * hidden row h the logits are z = h W^T, W holding one row of d weights per
+ * token; the call computes the statistics of rps_score_step (the same
+ * definitions, ties and output layout, slot r = hidden row r) without writing
+ * the logits to memory: a tensor-core contraction (bf16 x bf16, fp32
+ * accumulation) whose epilogue folds each tile of logits into the rows'
+ * softmax sums, maxima and top-k lists, then a merge launch.
+ * Layout: hidden [n_rows][d] and unembed [vocab][d], bf16, d contiguous, rows
+ * hidden_stride / unembed_stride elements apart (multiples of 8); bases 16-byte
+ * aligned; d a multiple of 64.
+ */
+typedef struct {
+    const void *hidden;
+    const void *unembed;
+    int32_t n_rows;
+    int32_t d;
+    int64_t vocab;
+    int64_t hidden_stride, unembed_stride;
+} rps_lmhead;
+
+/* Workspace bytes of rps_lmhead_row_stats (k_max 0 for statistics only); 0 for
+ * invalid arguments. The workspace needs no zeroing before its first use
+ * except its first 256 bytes (the health word of rps_workspace_init), so
+ * rps_workspace_init on the whole workspace is the simple rule. */
+size_t rps_lmhead_workspace_bytes(int32_t n_rows, int64_t vocab, int32_t k_max);
+
+/*
+ * Statistics of every hidden row's logits h W^T into `out` (top-k mode when
+ * out->topk_idx != NULL, with k = prm->k_max; prm may be NULL otherwise).
+ * d_logits_out: NULL normally; for testing, a device array [n_rows][vocab] of
+ * fp32 that also receives the logits the epilogue folds.
+ * Two launches on `stream`. Errors: RPS_ERR_INVALID_ARG for NULL pointers,
+ * sizes, strides or alignment out of range, or a small workspace;
+ * RPS_ERR_UNSUPPORTED for k_max above RPS_MAX_K; RPS_ERR_CUDA when the
+ * tensor-map encoder is not available. A bounded device wait that gives up
+ * reports RPS_DEVERR_TIMEOUT and leaves the workspace unhealthy, as for
+ * rps_score_step.
+ */
+rps_status rps_lmhead_row_stats(const rps_lmhead *lm, const rps_params *prm, const rps_row_stats *out,
+                                float *d_logits_out, void *d_ws, size_t ws_bytes, rps_stream_t stream);
+
 /* Synchronise `stream`, then read and clear the calling device's error word.
  * Returns RPS_OK or RPS_ERR_DEVICE (with the RPS_DEVERR_* bits in *detail when
  * detail != NULL), or RPS_ERR_CUDA if the synchronisation itself failed. */

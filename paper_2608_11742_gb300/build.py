@@ -23,10 +23,10 @@ FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcomp
                 f"-I{INCLUDE}", f"-I{CSRC}"]
 
 LIBS = {
-    "librps.so": ["abi.cu", "rowstats.cu", "decide.cu", "decode.cu", "gather.cu", "static_scratch.cu"],
+    "librps.so": ["abi.cu", "rowstats.cu", "decide.cu", "decode.cu", "gather.cu", "static_scratch.cu", "lmhead.cu"],
     "librps_synth.so": ["synth.cu"],
 }
-HEADERS = [INCLUDE / "rps.h", INCLUDE / "rps_synth.h", CSRC / "rps_internal.cuh"]
+HEADERS = [INCLUDE / "rps.h", INCLUDE / "rps_synth.h", CSRC / "rps_internal.cuh", CSRC / "umma_desc.h"]
 
 
 def _stale(target: Path, sources) -> bool:

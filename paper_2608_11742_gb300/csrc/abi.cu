@@ -119,6 +119,8 @@ uint32_t *device_error_word() {
     return device_info(&dev) == RPS_OK ? dev.err : nullptr;
 }
 
+uint64_t ring_wait_limit_ns() { return g_ring_wait_ns.load(std::memory_order_relaxed); }
+
 }  // namespace rps
 
 using namespace rps;

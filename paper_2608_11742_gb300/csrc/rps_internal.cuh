@@ -136,6 +136,9 @@ cudaError_t launch_score_commit(const ScoreArgs &s, const CommitArgs &c, cudaStr
 // The calling device's sticky error word (nullptr if the device cannot be queried).
 uint32_t *device_error_word();
 
+// The current limit of a kernel's wait for an asynchronous copy (rps_debug_set_ring_wait_ns).
+uint64_t ring_wait_limit_ns();
+
 // The host-side argument rules of rps_score_step (everything but the
 // workspace), checked before anything is enqueued; *k_out is the top-k size
 // (0 in statistics-only mode). Shared by every row-statistics entry point.

@@ -115,6 +115,16 @@ _lib.rps_status_string.restype = C.c_char_p
 _lib.rps_status_string.argtypes = [C.c_int]
 _lib.rps_version.restype = C.c_int32
 _lib.rps_version.argtypes = []
+class RpsLmhead(C.Structure):
+    _fields_ = [("hidden", _p), ("unembed", _p), ("n_rows", C.c_int32), ("d", C.c_int32), ("vocab", C.c_int64),
+                ("hidden_stride", C.c_int64), ("unembed_stride", C.c_int64)]
+
+
+_lib.rps_lmhead_workspace_bytes.restype = C.c_size_t
+_lib.rps_lmhead_workspace_bytes.argtypes = [C.c_int32, C.c_int64, C.c_int32]
+_lib.rps_lmhead_row_stats.restype = C.c_int
+_lib.rps_lmhead_row_stats.argtypes = [C.POINTER(RpsLmhead), C.POINTER(RpsParams), C.POINTER(RpsRowStats), _p, _p,
+                                      C.c_size_t, _p]
 _lib.rps_debug_set_ring_wait_ns.restype = C.c_uint64
 _lib.rps_debug_set_ring_wait_ns.argtypes = [C.c_uint64]
 
@@ -376,6 +386,31 @@ def rps_poll_device_status(stream=None):
     detail = C.c_uint32(0)
     st = _lib.rps_poll_device_status(_stream(stream), C.byref(detail))
     return st, detail.value
+
+
+def rps_lmhead_workspace_bytes(n_rows: int, vocab: int, k_max: int) -> int:
+    n = _lib.rps_lmhead_workspace_bytes(n_rows, vocab, k_max)
+    if n == 0:
+        raise RPSError(RPS_ERR_INVALID_ARG, "rps_lmhead_workspace_bytes")
+    return n
+
+
+def rps_lmhead_row_stats(hidden: torch.Tensor, unembed: torch.Tensor, prm, out: RowStatsBuf, ws: torch.Tensor,
+                         logits_out: Optional[torch.Tensor] = None, stream=None) -> None:
+    """Row statistics of ``hidden @ unembed.T`` (bf16 CUDA tensors ``[n][d]`` and
+    ``[V][d]``) into ``out``; ``logits_out`` (fp32 ``[n][V]``, testing) also
+    receives the logits."""
+    if hidden.dtype != torch.bfloat16 or unembed.dtype != torch.bfloat16:
+        raise TypeError("hidden and unembed must be bf16")
+    if hidden.dim() != 2 or unembed.dim() != 2 or hidden.stride(1) != 1 or unembed.stride(1) != 1:
+        raise ValueError("hidden [n][d] and unembed [V][d] with d contiguous")
+    lm = RpsLmhead(hidden.data_ptr(), unembed.data_ptr(), hidden.shape[0], hidden.shape[1], unembed.shape[0],
+                   hidden.stride(0), unembed.stride(0))
+    p = params(prm) if prm is not None else None
+    st = out.c()
+    _check(_lib.rps_lmhead_row_stats(C.byref(lm), None if p is None else C.byref(p), C.byref(st), _ptr(logits_out),
+                                     ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)),
+           "rps_lmhead_row_stats")
 
 
 # --------------------------------------------------------------------------- one step

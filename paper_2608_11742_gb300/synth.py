@@ -316,3 +316,15 @@ def device_advance(winner, B: int, L_total: int, d_block, d_step, scale, epoch, 
                                         stream.cuda_stream)
     if rc != 0:
         raise RuntimeError(f"rps_synth_advance failed with code {rc}")
+
+
+def lmhead_inputs(seed: int, n_rows: int, V: int, d: int, logit_scale: float = 3.0):
+    """Seeded LM-head operands as bf16 bits (uint16): hidden [n_rows][d] with
+    unit-variance entries, and an unembedding [V][d] whose entries have standard
+    deviation logit_scale / sqrt(d), so that the logits h W^T spread over about
+    logit_scale nats per standard deviation. numpy's PCG64 normal generator."""
+    rng = np.random.default_rng(seed)
+    h = rng.standard_normal((n_rows, d), dtype=np.float32)
+    w = rng.standard_normal((V, d), dtype=np.float32)
+    w *= np.float32(logit_scale / np.sqrt(d))
+    return bf16_round(h), bf16_round(w)
