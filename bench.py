@@ -55,6 +55,8 @@ OTHERS = ("step", "step-50", "step-10", "long", "block", "tiny")
 REPLAY_STEPS = 64
 FLUSH_BYTES = 256 << 20
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+LMHEAD_D = 4096  # hidden size of the 126,464-token model
 KERNEL_SOURCES = ("paper_2608_11742_gb300/csrc/rowstats.cu", "paper_2608_11742_gb300/csrc/rps_internal.cuh")
 
 
@@ -105,6 +107,14 @@ def peaks():
         d = json.loads(p.read_text())
         return float(d["hbm_gbs"]), "measured"
     return FALLBACK_HBM_GBS, "fallback"
+
+
+def tensor_peak():
+    """Dense bf16 tensor-core peak (TFLOP/s) for a kernel timed alone: the measured burst figure."""
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        return float(json.loads(p.read_text())["bf16_tflops"]), "measured"
+    return FALLBACK_BF16_TFLOPS, "fallback"
 
 
 def dist_env():
@@ -407,6 +417,74 @@ def long_replay(configs, device, flush, peak: float) -> dict:
                       "advance of the generator and the mask run outside the timed region"}
 
 
+def lmhead_run(configs, device, flush, steps: int, warmup: int) -> dict:
+    """The LM head with the statistics in its epilogue (rps_lmhead_row_stats) on
+    the step workload's scored rows: 256 base rows in top-k mode (k 10) and
+    1,152 lookahead rows statistics-only, hidden size 4,096, vocabulary 126,464.
+    Random bf16 operands (seeded); each launch is timed alone with CUDA events
+    after an L2 flush. cuBLAS (torch.matmul to bf16 logits) on the same shapes is
+    timed beside it for context: it writes the logits the fused kernel never does."""
+    import torch
+    from paper_2608_11742_gb300 import rps
+    w = configs.STEP
+    prm = w.params(configs.EXERCISE)
+    peak_tf, peak_kind = tensor_peak()
+    hbm, _ = peaks()
+    V, d = w.V, LMHEAD_D
+    g = torch.Generator(device=device)
+    g.manual_seed(7)
+    W = (torch.randn((V, d), generator=g, device=device) * (3.0 / d ** 0.5)).to(torch.bfloat16)
+    parts = {"base rows (top-k)": (256, prm.k_max), "lookahead rows (statistics)": (1152, 0)}
+    out = {"workload": f"{sum(n for n, _ in parts.values())} scored rows of the step workload, hidden size {d}, "
+                       f"vocabulary {V}, bf16 operands (seeded random), fp32 accumulation",
+           "peak_tflops": peak_tf, "peak_kind": peak_kind, "launches": {}}
+    stream = torch.cuda.Stream(device)
+    total_ms = total_flop = 0.0
+    for name, (n, k) in parts.items():
+        h = torch.randn((n, d), generator=g, device=device).to(torch.bfloat16)
+        buf = rps.RowStatsBuf.alloc(n, k, device)
+        ws = torch.empty(rps.rps_lmhead_workspace_bytes(n, V, k), dtype=torch.uint8, device=device)
+        rps.rps_workspace_init(ws)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+        def timed(fn):
+            ms = []
+            for i in range(warmup + steps):
+                with torch.cuda.stream(stream):
+                    flush()
+                    e0.record(stream)
+                    fn()
+                    e1.record(stream)
+                stream.synchronize()
+                if i >= warmup:
+                    ms.append(e0.elapsed_time(e1))
+            return statistics.mean(ms)
+
+        t = timed(lambda: rps.rps_lmhead_row_stats(h, W, prm if k else None, buf, ws))
+        st, detail = rps.rps_poll_device_status(stream)
+        if st != rps.RPS_OK:
+            raise RuntimeError(f"lmhead device error {detail:#x}")
+        t_cublas = timed(lambda: torch.matmul(h, W.t()))
+        flop = 2.0 * n * d * V
+        tf = flop / (t / 1e3) / 1e12
+        out["launches"][name] = {
+            "rows": n, "k": k, "ms": t, "tflops": tf, "frac_of_tensor_peak": tf / peak_tf,
+            "unembedding_gbs": V * d * 2 / (t / 1e3) / 1e9, "unembedding_frac_of_hbm": V * d * 2 / (t / 1e3) / 1e9 / hbm,
+            "cublas_matmul_ms": t_cublas, "cublas_tflops": flop / (t_cublas / 1e3) / 1e12,
+            "logit_bytes_not_written": n * V * 2}
+        total_ms += t
+        total_flop += flop
+        del h, buf, ws
+    out["step_ms"] = total_ms
+    out["tflops"] = total_flop / (total_ms / 1e3) / 1e12
+    out["frac_of_tensor_peak"] = out["tflops"] / peak_tf
+    out["roofline"] = {"bound": "tensor", "kernel": "lmhead_kernel (tcgen05) + merge, both launches",
+                       "achieved": out["tflops"], "peak": peak_tf, "unit": "TFLOP/s", "frac": out["frac_of_tensor_peak"],
+                       "algorithmic_flop_per_step": total_flop}
+    del W
+    return out
+
+
 def decode_run(configs, device):
     """A whole response decoded on the device (Algorithm 1): the block workload's
     64 requests x 32-position blocks extended to 256 positions. The denoiser
@@ -569,6 +647,10 @@ def run_gpu(args):
         out["decode"] = decode_run(configs, device)
         torch.cuda.empty_cache()
 
+    if not args.skip_lmhead:
+        out["lmhead"] = lmhead_run(configs, device, flush, max(5, args.steps // 2), 3)
+        torch.cuda.empty_cache()
+
     if not args.skip_e2e:
         wl = Workload(w, prm, device)
         ms, h2d, d2h, ms_full, h2d_full = wl.e2e(max(3, args.steps // 4), 3)
@@ -632,6 +714,9 @@ def main():
     ap.add_argument("--skip-others", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--skip-decode", action="store_true")
+    ap.add_argument("--skip-lmhead", action="store_true")
+    ap.add_argument("--only-lmhead", action="store_true",
+                    help="time the LM head with the statistics epilogue alone and print its record")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()
@@ -639,6 +724,12 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.only_lmhead:
+        import torch
+        from paper_2608_11742_gb300 import configs
+        device = torch.device("cuda", dist_env()[2])
+        torch.cuda.set_device(device)
+        print(json.dumps({"lmhead": lmhead_run(configs, device, L2Flush(device), args.steps, args.warmup)}))
     else:
         run_gpu(args)
 
