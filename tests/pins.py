@@ -768,10 +768,108 @@ def pin_lmhead_token_permutation(o):
     close(b.H, a.H, tol=1e-12, what="H")
 
 
+def _attn_case(seed, n_b, n_h, C, NB, G, D, spread=1.0):
+    rng = np.random.default_rng(seed)
+    n = C + NB * G
+    return tuple(synth.bf16_round((rng.standard_normal((n_b, n_h, n, D)) * spread).astype(np.float32))
+                 for _ in range(3))
+
+
+def _bits_f64(b):
+    return (np.asarray(b, np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def pin_attention_dense_mask(o):
+    """The packed attention equals masked softmax attention under the dense
+    token-by-token mask written out from the isolation rule (a key is visible
+    when it is a context token or lies in the query's own branch; context
+    queries own branch 0), for every query at once."""
+    from oracle.attention import packed_attention
+    C, NB, G, D, scale = 5, 3, 4, 8, 0.37
+    q, k, v = _attn_case(21, 2, 2, C, NB, G, D)
+    out = packed_attention(q, k, v, C, NB, G, scale)
+    seg = np.array([0] * C + [1 + j for j in range(NB) for _ in range(G)])
+    own = np.where(seg == 0, 1, seg)
+    visible = (seg[None, :] == 0) | (seg[None, :] == own[:, None])
+    qf, kf, vf = _bits_f64(q), _bits_f64(k), _bits_f64(v)
+    for b in range(2):
+        for h in range(2):
+            s = scale * qf[b, h] @ kf[b, h].T
+            s = np.where(visible, s, -np.inf)
+            p = np.exp(s - s.max(axis=1, keepdims=True))
+            p /= p.sum(axis=1, keepdims=True)
+            close(out[b, h], p @ vf[b, h], tol=1e-12, what="dense-mask attention")
+
+
+def pin_attention_branch_is_plain_attention(o):
+    """Each branch's queries get exactly plain (unmasked) attention over the
+    sequence [context, that branch], and the context's queries plain attention
+    over [context, branch 0]: a library routine (torch's scaled dot-product
+    attention, fp64) on the unpacked sequence."""
+    import torch
+    from oracle.attention import packed_attention
+    C, NB, G, D = 6, 4, 5, 16
+    scale = 1.0 / math.sqrt(D)
+    q, k, v = _attn_case(22, 1, 3, C, NB, G, D, spread=2.0)
+    out = packed_attention(q, k, v, C, NB, G, scale)
+    qf, kf, vf = (torch.from_numpy(_bits_f64(x)) for x in (q, k, v))
+    for j in range(NB):
+        idx = list(range(C)) + list(range(C + j * G, C + (j + 1) * G))
+        ref = torch.nn.functional.scaled_dot_product_attention(qf[:, :, idx], kf[:, :, idx], vf[:, :, idx]).numpy()
+        close(out[:, :, C + j * G:C + (j + 1) * G], ref[:, :, C:], tol=1e-12, what=f"branch {j}")
+        if j == 0:
+            close(out[:, :, :C], ref[:, :, :C], tol=1e-12, what="context")
+
+
+def pin_attention_isolation(o):
+    """Changing one branch's keys and values changes that branch's outputs
+    only: the context and every other branch are bit-identical."""
+    from oracle.attention import packed_attention
+    C, NB, G, D = 4, 4, 3, 8
+    q, k, v = _attn_case(23, 1, 2, C, NB, G, D)
+    base = packed_attention(q, k, v, C, NB, G, 0.5)
+    k2, v2 = k.copy(), v.copy()
+    rows = slice(C + 2 * G, C + 3 * G)
+    k2[:, :, rows] = synth.bf16_round(np.random.default_rng(24).standard_normal(k2[:, :, rows].shape).astype(np.float32))
+    v2[:, :, rows] = synth.bf16_round(np.random.default_rng(25).standard_normal(v2[:, :, rows].shape).astype(np.float32))
+    moved = packed_attention(q, k2, v2, C, NB, G, 0.5)
+    keep = np.ones(C + NB * G, bool)
+    keep[rows] = False
+    assert np.array_equal(base[:, :, keep], moved[:, :, keep]), "another branch saw branch 2"
+    assert not np.allclose(base[:, :, rows], moved[:, :, rows]), "branch 2 ignores its own keys"
+
+
+def pin_attention_closed_forms(o):
+    """Identical keys give uniform weights: the output is the mean of the
+    visible values. A key whose score leads every other by 60 nats gives its
+    own value."""
+    from oracle.attention import packed_attention
+    C, NB, G, D = 3, 3, 2, 4
+    q, k, v = _attn_case(26, 1, 1, C, NB, G, D)
+    k[:] = k[:, :, :1]
+    out = packed_attention(q, k, v, C, NB, G, 0.8)
+    vf = _bits_f64(v)[0, 0]
+    for j in range(NB):
+        vis = list(range(C)) + list(range(C + j * G, C + (j + 1) * G))
+        close(out[0, 0, C + j * G:C + (j + 1) * G], np.broadcast_to(vf[vis].mean(axis=0), (G, D)), tol=1e-12,
+              what=f"uniform weights, branch {j}")
+    close(out[0, 0, :C], np.broadcast_to(vf[list(range(C + G))].mean(axis=0), (C, D)), tol=1e-12, what="context")
+    # one dominant key in branch 1 (token C + G + 1): q . k = 60 / scale more than any other
+    q2, k2, v2 = _attn_case(27, 1, 1, C, NB, G, D)
+    qf = np.zeros((1, 1, C + NB * G, D))
+    qf[..., 0] = 1.0
+    kf = np.zeros_like(qf)
+    kf[0, 0, C + G + 1, 0] = 60.0
+    out = packed_attention(_bf16_bits(qf), _bf16_bits(kf), v2, C, NB, G, 1.0)
+    close(out[0, 0, C + G:C + 2 * G], np.broadcast_to(_bits_f64(v2)[0, 0, C + G + 1], (G, D)), tol=1e-20,
+          what="dominant key")
+
+
 ALL_PINS = [
     pin_uniform_rows, pin_spike_rows, pin_two_level_rows, pin_rank_order, pin_library_crosscheck,
     pin_synth_rows_crosscheck, pin_invariants, pin_neg_inf_entries, pin_select_brute_force,
     pin_score_commit_brute_force, pin_score_closed_form, pin_control_flow, pin_exact_thresholds,
     pin_propositions, pin_lmhead_worked_example, pin_lmhead_zero_hidden, pin_lmhead_token_shift,
-    pin_lmhead_token_permutation,
+    pin_lmhead_token_permutation, pin_attention_dense_mask, pin_attention_branch_is_plain_attention,
+    pin_attention_isolation, pin_attention_closed_forms,
 ]

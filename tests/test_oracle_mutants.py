@@ -115,3 +115,33 @@ def test_lmhead_mutant_is_caught(oracle, monkeypatch, name):
             caught = True
             break
     assert caught, f"no LM-head pin catches '{name}'"
+
+
+# Planted mistakes in the packed-attention oracle: each must fail an attention pin.
+def _attn_mutants():
+    import numpy as np
+    import oracle.attention as at
+    keys, soft = at.allowed_keys, at.softmax_attention
+    return {
+        "context sees every branch": ("allowed_keys", lambda C, NB, G, s: np.arange(C + NB * G) if s == 0 else keys(C, NB, G, s)),
+        "branch sees the next branch": ("allowed_keys", lambda C, NB, G, s: keys(C, NB, G, s if s in (0, NB) else s + 1)),
+        "last context key dropped": ("allowed_keys", lambda C, NB, G, s: keys(C, NB, G, s)[1:]),
+        "scale dropped": ("softmax_attention", lambda q, k, v, scale: soft(q, k, v, 1.0)),
+        "keys for values": ("softmax_attention", lambda q, k, v, scale: soft(q, k, k, scale)),
+    }
+
+
+@pytest.mark.parametrize("name", ["context sees every branch", "branch sees the next branch", "last context key dropped",
+                                  "scale dropped", "keys for values"])
+def test_attention_mutant_is_caught(oracle, monkeypatch, name):
+    import oracle.attention as at
+    attr, fn = _attn_mutants()[name]
+    monkeypatch.setattr(at, attr, fn)
+    caught = False
+    for pin in (p for p in pins.ALL_PINS if p.__name__.startswith("pin_attention")):
+        try:
+            pin(oracle)
+        except Exception:
+            caught = True
+            break
+    assert caught, f"no attention pin catches '{name}'"
