@@ -485,6 +485,65 @@ def lmhead_run(configs, device, flush, steps: int, warmup: int) -> dict:
     return out
 
 
+def attention_run(device, flush, steps: int, warmup: int) -> dict:
+    """The branch-isolating attention of the packed lookahead forward pass
+    (rps_packed_attention_fwd) at the serving shape: 8 requests x 32 heads x
+    head dim 128, a 512-token context and the anchor plus 8 branches of the
+    256-token generation region (2,816 packed tokens). Random bf16 inputs
+    (seeded); CUDA events after an L2 flush. torch's scaled-dot-product
+    attention with the same mask written out densely is timed for context."""
+    import torch
+    from paper_2608_11742_gb300 import rps
+    B, H, D, C, NB, G = 8, 32, 128, 512, 9, 256
+    n = C + NB * G
+    g = torch.Generator(device=device)
+    g.manual_seed(9)
+    q, k, v = (torch.randn((B, H, n, D), generator=g, device=device).to(torch.bfloat16) for _ in range(3))
+    vt = v.transpose(2, 3).contiguous()
+    out = torch.empty_like(q)
+    scale = D ** -0.5
+    stream = torch.cuda.Stream(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn):
+        ms = []
+        for i in range(warmup + steps):
+            with torch.cuda.stream(stream):
+                flush()
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+            stream.synchronize()
+            if i >= warmup:
+                ms.append(e0.elapsed_time(e1))
+        return statistics.mean(ms)
+
+    t = timed(lambda: rps.rps_packed_attention_fwd(q, k, vt, out, C, NB, G, scale))
+    st, detail = rps.rps_poll_device_status(stream)
+    if st != rps.RPS_OK:
+        raise RuntimeError(f"attention device error {detail:#x}")
+    pairs = C * (C + G) + NB * G * (C + G)  # visible (query, key) pairs per head
+    flop = 4.0 * D * B * H * pairs
+    peak_tf, peak_kind = tensor_peak()
+    tf = flop / (t / 1e3) / 1e12
+    rec = {"workload": f"{B} requests x {H} heads x head dim {D}: context {C} + {NB} branches (anchor and "
+                       f"{NB - 1} candidates) x {G} tokens = {n} packed tokens, bf16",
+           "ms": t, "tflops": tf, "frac_of_tensor_peak": tf / peak_tf, "peak_tflops": peak_tf, "peak_kind": peak_kind,
+           "algorithmic_flop": flop, "visible_fraction_of_dense": pairs / (n * n),
+           "roofline": {"bound": "tensor", "kernel": "packed_attention_kernel (tcgen05)", "achieved": tf,
+                        "peak": peak_tf, "unit": "TFLOP/s", "frac": tf / peak_tf}}
+    seg = torch.cat([torch.zeros(C, dtype=torch.int64)] + [torch.full((G,), 1 + j) for j in range(NB)]).to(device)
+    own = torch.where(seg == 0, torch.ones_like(seg), seg)
+    mask = (seg[None, :] == 0) | (seg[None, :] == own[:, None])
+    try:
+        t_sdpa = timed(lambda: torch.nn.functional.scaled_dot_product_attention(q, k, v, attn_mask=mask))
+        rec["torch_sdpa_dense_mask_ms"] = t_sdpa
+    except RuntimeError as exc:  # no kernel for this mask / size
+        rec["torch_sdpa_dense_mask_ms"] = f"unavailable: {exc}"[:200]
+    del q, k, v, vt, out, mask
+    return rec
+
+
 def decode_run(configs, device):
     """A whole response decoded on the device (Algorithm 1): the block workload's
     64 requests x 32-position blocks extended to 256 positions. The denoiser
@@ -650,6 +709,8 @@ def run_gpu(args):
     if not args.skip_lmhead:
         out["lmhead"] = lmhead_run(configs, device, flush, max(5, args.steps // 2), 3)
         torch.cuda.empty_cache()
+        out["attention"] = attention_run(device, flush, max(5, args.steps // 2), 3)
+        torch.cuda.empty_cache()
 
     if not args.skip_e2e:
         wl = Workload(w, prm, device)
@@ -716,7 +777,8 @@ def main():
     ap.add_argument("--skip-decode", action="store_true")
     ap.add_argument("--skip-lmhead", action="store_true")
     ap.add_argument("--only-lmhead", action="store_true",
-                    help="time the LM head with the statistics epilogue alone and print its record")
+                    help="time the tensor-core extensions alone (LM head with the statistics epilogue, packed "
+                         "lookahead attention) and print their records")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()
@@ -729,7 +791,9 @@ def main():
         from paper_2608_11742_gb300 import configs
         device = torch.device("cuda", dist_env()[2])
         torch.cuda.set_device(device)
-        print(json.dumps({"lmhead": lmhead_run(configs, device, L2Flush(device), args.steps, args.warmup)}))
+        flush = L2Flush(device)
+        print(json.dumps({"lmhead": lmhead_run(configs, device, flush, args.steps, args.warmup),
+                          "attention": attention_run(device, flush, args.steps, args.warmup)}))
     else:
         run_gpu(args)
 

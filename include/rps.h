@@ -423,6 +423,38 @@ size_t rps_lmhead_workspace_bytes(int32_t n_rows, int64_t vocab, int32_t k_max);
 rps_status rps_lmhead_row_stats(const rps_lmhead *lm, const rps_params *prm, const rps_row_stats *out,
                                 float *d_logits_out, void *d_ws, size_t ws_bytes, rps_stream_t stream);
 
+/*
+ * Branch-isolating attention of the packed lookahead forward pass (Sec. 3.1
+ * "Lookahead scoring"; Fig. 2, right). The lookahead pass scores all branches
+ * of a step in one forward pass over a packed sequence of n_tokens =
+ * n_context + n_branch * branch_len tokens: the shared context, then the
+ * generation region once per branch (branch 0 = the anchor, the normal
+ * sequence's own region). A query of branch j attends to the context and to
+ * branch j only; a context query attends to the context and branch 0 (the
+ * normal sequence). For every (batch, head):
+ *   out_i = sum_{k visible from i} softmax_k(scale * q_i . k_k) v_k
+ * bf16 inputs and output, fp32 scores and accumulation, probabilities rounded
+ * to bf16 before they weight the values. No dense mask is formed.
+ * Layout (bf16, contiguous): q, k, out [n_batch][n_heads][n_tokens][head_dim];
+ * vt [n_batch][n_heads][head_dim][n_tokens] (the values transposed, tokens
+ * contiguous). head_dim must be 128; n_context (>= 0) and branch_len (>= 1)
+ * multiples of 8; bases 16-byte aligned.
+ */
+typedef struct {
+    const void *q, *k, *vt;
+    void *out;
+    int32_t n_batch, n_heads, head_dim;
+    int32_t n_context, n_branch, branch_len;
+    float scale;
+} rps_packed_attention;
+
+/* One launch on `stream`. Errors: RPS_ERR_INVALID_ARG for NULL or misaligned
+ * pointers and sizes out of range; RPS_ERR_UNSUPPORTED for head_dim != 128 or
+ * tensors above 2^31 rows; RPS_ERR_CUDA when the tensor-map encoder is not
+ * available. A bounded device wait that gives up reports RPS_DEVERR_TIMEOUT
+ * (the output is then incomplete). */
+rps_status rps_packed_attention_fwd(const rps_packed_attention *attn, rps_stream_t stream);
+
 /* Synchronise `stream`, then read and clear the calling device's error word.
  * Returns RPS_OK or RPS_ERR_DEVICE (with the RPS_DEVERR_* bits in *detail when
  * detail != NULL), or RPS_ERR_CUDA if the synchronisation itself failed. */

@@ -23,7 +23,7 @@ FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcomp
                 f"-I{INCLUDE}", f"-I{CSRC}"]
 
 LIBS = {
-    "librps.so": ["abi.cu", "rowstats.cu", "decide.cu", "decode.cu", "gather.cu", "static_scratch.cu", "lmhead.cu"],
+    "librps.so": ["abi.cu", "rowstats.cu", "decide.cu", "decode.cu", "gather.cu", "static_scratch.cu", "lmhead.cu", "attention.cu"],
     "librps_synth.so": ["synth.cu"],
 }
 HEADERS = [INCLUDE / "rps.h", INCLUDE / "rps_synth.h", CSRC / "rps_internal.cuh", CSRC / "umma_desc.h"]

@@ -208,6 +208,13 @@ __device__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Ctl &c, const LmAr
 }
 
 // A wait that only ends early when the phase completes (drains before exit).
+// wait_or_abort for every lane of a warp that goes on to warp-wide tcgen05
+// instructions: the warp leaves together, on the same answer.
+template <typename Ctl_, typename Args_>
+__device__ __forceinline__ bool warp_wait_or_abort(uint64_t *bar, uint32_t parity, Ctl_ &c, const Args_ &a) {
+    return __all_sync(kFull, wait_or_abort(bar, parity, c, a));
+}
+
 __device__ void wait_drain(uint64_t *bar, uint32_t parity) {
     if (mbar_try_wait(bar, parity)) return;
     const uint64_t start = global_ns();
@@ -367,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < n_tiles; ++t) {
             const int buf = t & 1;
             const uint32_t use = static_cast<uint32_t>(t >> 1);
-            if (!wait_or_abort(&c.acc_full[buf], use & 1, c, a)) {
+            if (!warp_wait_or_abort(&c.acc_full[buf], use & 1, c, a)) {
                 ok = false;
                 break;
             }

@@ -125,6 +125,14 @@ _lib.rps_lmhead_workspace_bytes.argtypes = [C.c_int32, C.c_int64, C.c_int32]
 _lib.rps_lmhead_row_stats.restype = C.c_int
 _lib.rps_lmhead_row_stats.argtypes = [C.POINTER(RpsLmhead), C.POINTER(RpsParams), C.POINTER(RpsRowStats), _p, _p,
                                       C.c_size_t, _p]
+class RpsPackedAttention(C.Structure):
+    _fields_ = [("q", _p), ("k", _p), ("vt", _p), ("out", _p), ("n_batch", C.c_int32), ("n_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("n_context", C.c_int32), ("n_branch", C.c_int32),
+                ("branch_len", C.c_int32), ("scale", C.c_float)]
+
+
+_lib.rps_packed_attention_fwd.restype = C.c_int
+_lib.rps_packed_attention_fwd.argtypes = [C.POINTER(RpsPackedAttention), _p]
 _lib.rps_debug_set_ring_wait_ns.restype = C.c_uint64
 _lib.rps_debug_set_ring_wait_ns.argtypes = [C.c_uint64]
 
@@ -411,6 +419,23 @@ def rps_lmhead_row_stats(hidden: torch.Tensor, unembed: torch.Tensor, prm, out: 
     _check(_lib.rps_lmhead_row_stats(C.byref(lm), None if p is None else C.byref(p), C.byref(st), _ptr(logits_out),
                                      ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream)),
            "rps_lmhead_row_stats")
+
+
+def rps_packed_attention_fwd(q: torch.Tensor, k: torch.Tensor, vt: torch.Tensor, out: torch.Tensor, n_context: int,
+                             n_branch: int, branch_len: int, scale: float, stream=None) -> None:
+    """Branch-isolating attention of a packed lookahead sequence: q, k, out
+    ``[batch][heads][tokens][128]`` and vt ``[batch][heads][128][tokens]``, bf16 CUDA tensors."""
+    for t in (q, k, vt, out):
+        if t.dtype != torch.bfloat16 or not t.is_contiguous() or t.dim() != 4:
+            raise ValueError("q, k, vt and out must be contiguous 4-D bf16 tensors")
+    n_b, n_h, n_tok, d = q.shape
+    if k.shape != q.shape or out.shape != q.shape or vt.shape != (n_b, n_h, d, n_tok):
+        raise ValueError("shapes: q, k, out [b][h][tokens][d] and vt [b][h][d][tokens]")
+    if n_tok != n_context + n_branch * branch_len:
+        raise ValueError("tokens must be n_context + n_branch * branch_len")
+    a = RpsPackedAttention(q.data_ptr(), k.data_ptr(), vt.data_ptr(), out.data_ptr(), n_b, n_h, d, n_context,
+                           n_branch, branch_len, scale)
+    _check(_lib.rps_packed_attention_fwd(C.byref(a), _stream(stream)), "rps_packed_attention_fwd")
 
 
 # --------------------------------------------------------------------------- one step
