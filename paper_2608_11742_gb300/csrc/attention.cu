@@ -11,10 +11,12 @@
 // the keys past its end.
 //
 // One persistent CTA per SM takes work items (batch, head, 128-query tile):
-//   warp 0      TMA producer: the Q tile (128 x 128, two 64-wide swizzle
-//               atoms), then per key tile K (128 keys x 128) and V^T (128 dims
-//               x 128 keys; V is stored transposed so that both MMA operands
-//               are K-major), 128-byte swizzle, two stages;
+//   warp 0      TMA producer of Q (128 x 128, two 64-wide swizzle atoms) and,
+//               per key tile, K (128 keys x 128), 128-byte swizzle, two stages;
+//   warp 6      TMA producer of V^T (128 dims x 128 keys: V is stored
+//               transposed so that both MMA operands are K-major), two stages
+//               of their own, so that K runs ahead of V (K is free once S is
+//               computed, V only once P V is);
 //   warp 1      MMA issuer: S = Q K^T (M 128, N 128, K 128) into one of two
 //               TMEM buffers, then O += P V^T into the TMEM accumulator once
 //               the softmax has written P; it also allocates and frees TMEM;
@@ -22,8 +24,9 @@
 //               finds the tile maximum; the base-2 reference m is raised only
 //               when a score passes it by more than 8 (then O and the running
 //               sum are rescaled in TMEM); pass 2 writes P = 2^(s c - m) as bf16
-//               into shared memory in the swizzled layout the MMA reads. At the
-//               end of an item O / l is written to global memory as bf16.
+//               into one of two shared-memory buffers, in the swizzled layout
+//               the MMA reads, while the MMA still reads the other. At the end
+//               of an item O / l is written to global memory as bf16.
 // Every wait is bounded; a role whose wait runs out flags RPS_DEVERR_TIMEOUT
 // and raises the CTA's abort flag, copies and MMAs in flight are drained and
 // TMEM is freed before the CTA exits.
@@ -49,14 +52,14 @@ constexpr int kAtom = 64 * 128 * 2;          // one 128-row x 64-column bf16 swi
 constexpr int kQBytes = 2 * kAtom;           // Q tile: two atoms along d
 constexpr int kKBytes = 2 * kAtom;           // K tile: two atoms along d
 constexpr int kVBytes = 2 * kAtom;           // V^T tile: two atoms along the keys
-constexpr int kPBytes = 2 * kAtom;           // P tile: two atoms along the keys
 constexpr int kKvStages = 2;
-constexpr int kKvBytes = kKBytes + kVBytes;
-constexpr int kSmemBytes = kQBytes + kKvStages * kKvBytes + kPBytes + 1024;
-constexpr int kThreads = 192;
-constexpr int kSoftWarps = 4;
-constexpr uint32_t kTmemCols = 512;          // S buffers at columns 0 and 128, O at 256
-constexpr uint32_t kOCol = 256;
+constexpr int kPBufs = 2;                    // P of tile j lives in TMEM, in place of S buffer j % 2
+constexpr int kSmemBytes = kQBytes + kKvStages * (kKBytes + kVBytes) + 1024;
+constexpr int kThreads = 352;                // warp 0 and 10 TMA, warp 1 MMA, warps 2-9 softmax
+constexpr int kSoftWarps = 8;                // two per TMEM lane quarter: one per half of the keys
+constexpr int kVWarp = 10;
+constexpr uint32_t kTmemCols = 512;          // S buffers at columns 0 and 128, O buffers at 256 and 384
+constexpr uint32_t kOCol = 256;              // O of item n at kOCol + (n % 2) * kD
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescale = 8.0f;             // base-2 units a score may pass the reference by
 constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
@@ -125,6 +128,28 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
         "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+// D[tmem] (+)= A[tmem] x B[smem]^T: the A operand (128 rows x 16 bf16, two per
+// 32-bit column, lane = row) read from tensor memory.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_st32_u(uint32_t taddr, const uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
+        "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),
+        "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(saddr(bar))
                  : "memory");
@@ -144,6 +169,52 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
+// 32 columns without waiting: the registers are valid only after tmem_wait_dep on them.
+__device__ __forceinline__ void tmem_ld32_async(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+}
+// Waits for this thread's outstanding tcgen05.ld; naming the registers as
+// operands keeps every later use of them after the wait.
+__device__ __forceinline__ void tmem_wait_dep(uint32_t (&r)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                   "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                   "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+                 :
+                 : "memory");
+}
+
+// Packed fp32 pairs (one instruction for two lanes of work).
+typedef unsigned long long f2;
+__device__ __forceinline__ f2 pack2(float lo, float hi) {
+    f2 r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void unpack2(f2 v, float &lo, float &hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ f2 fma2(f2 a, f2 b, f2 c) {
+    f2 r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ f2 add2(f2 a, f2 b) {
+    f2 r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
@@ -216,7 +287,11 @@ __device__ __forceinline__ void key_tile(const AttnArgs &a, const Item &it, int 
 }
 
 struct Ctl {
-    uint64_t q_full, q_empty, kv_full[kKvStages], kv_empty[kKvStages], s_full[2], p_full, pv_done, o_free, mma_done;
+    uint64_t q_full, q_empty, k_full[kKvStages], k_empty[kKvStages], v_full[kKvStages], v_empty[kKvStages];
+    uint64_t s_full[2], p_full, pv_done[kPBufs], o_free[2], mma_done;
+    // the two halves of a row trade their tile maxima and, at the end of an
+    // item, their sums: (stamp << 32 | value bits), double-buffered by parity
+    uint64_t xmax[2][2][kBQ], xsum[2][2][kBQ];  // [parity][half][row]
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -248,6 +323,98 @@ __device__ void wait_drain(uint64_t *bar, uint32_t parity) {
         if (mbar_try_wait(bar, parity)) return;
 }
 
+// Waits (warp-wide) for the P V product of global key tile x, unless an
+// earlier wait already covered it. pv_done[x % 2] completes one phase per
+// product that reads P buffer x % 2; waited[b] counts the phases this thread
+// has seen, and a product is only waited for before the one two tiles later
+// can have been issued, so the parity names one phase.
+__device__ __forceinline__ bool wait_pv(uint32_t x, uint32_t (&waited)[kPBufs], Ctl &c, const AttnArgs &a) {
+    const uint32_t b = x & 1, ph = x >> 1;
+    if (waited[b] > ph) return true;
+    if (!warp_wait_or_abort(&c.pv_done[b], ph & 1, c, a)) return false;
+    waited[b] = ph + 1;
+    return true;
+}
+
+// Publishes this half-row's value for the partner half (stamp != 0).
+__device__ __forceinline__ void xput(uint64_t *slot, uint32_t stamp, float v) {
+    const uint64_t x = (static_cast<uint64_t>(stamp) << 32) | __float_as_uint(v);
+    asm volatile("st.volatile.shared.u64 [%0], %1;" ::"r"(saddr(slot)), "l"(x) : "memory");
+}
+
+// The partner half's value with `stamp`, bounded like every other wait; the
+// warp leaves together (false: the CTA aborts).
+__device__ bool xget(uint64_t *slot, uint32_t stamp, float &v, Ctl &c, const AttnArgs &a) {
+    uint64_t x = 0;
+    bool ok = false;
+    const uint64_t start = global_ns();
+    for (uint32_t n = 0;; ++n) {
+        asm volatile("ld.volatile.shared.u64 %0, [%1];" : "=l"(x) : "r"(saddr(slot)) : "memory");
+        if (static_cast<uint32_t>(x >> 32) == stamp) {
+            ok = true;
+            break;
+        }
+        if (*reinterpret_cast<volatile int *>(&c.abort_flag)) break;
+        if ((n & 63) == 63 && (a.wait_ns == 0 || global_ns() - start > a.wait_ns)) {
+            flag_error(a.err, RPS_DEVERR_TIMEOUT);
+            *reinterpret_cast<volatile int *>(&c.abort_flag) = 1;
+            break;
+        }
+    }
+    v = __uint_as_float(static_cast<uint32_t>(x));
+    return __all_sync(kFull, ok);
+}
+
+// An item whose O still waits to be written out.
+struct Pending {
+    bool active;
+    Item it;
+    float l;
+    uint32_t glast, ocol;
+    int n;
+};
+
+// O / l of this thread's half-row of a finished item (64 of the 128 columns),
+// bf16, to global memory; then the item's O buffer is released to the MMA
+// (o_free of its parity). The row sum is the two halves' sums added in a
+// fixed order.
+__device__ bool read_out(const Pending &pd, uint32_t (&waited)[kPBufs], uint32_t tmem, uint32_t lane_off, int r,
+                         int h, int lane, Ctl &c, const AttnArgs &a) {
+    if (!wait_pv(pd.glast, waited, c, a)) return false;
+    tc_fence_after();
+    const uint32_t stamp = static_cast<uint32_t>(pd.n) + 1u;
+    xput(&c.xsum[pd.n & 1][h][r], stamp, pd.l);
+    float other;
+    if (!xget(&c.xsum[pd.n & 1][h ^ 1][r], stamp, other, c, a)) return false;
+    const float l = h == 0 ? pd.l + other : other + pd.l;
+    const bool live = r < pd.it.q_len;
+    const float inv = 1.f / l;
+    __nv_bfloat16 *dst = a.out + (static_cast<int64_t>(pd.it.bh) * a.n_tokens + pd.it.q_start + r) * kD + h * 64;
+    uint32_t o[2][32];
+#pragma unroll
+    for (int ch = 0; ch < 2; ++ch) tmem_ld32_async(tmem + lane_off + pd.ocol + h * 64 + ch * 32, o[ch]);
+#pragma unroll
+    for (int ch = 0; ch < 2; ++ch) tmem_wait_dep(o[ch]);
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&c.o_free[pd.n & 1]);  // the buffer may take item n + 2
+    if (live) {
+#pragma unroll
+        for (int ch = 0; ch < 2; ++ch) {
+            uint4 *d4 = reinterpret_cast<uint4 *>(dst + ch * 32);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const uint32_t *x = o[ch] + 8 * u;
+                d4[u] = make_uint4(pack_bf16(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv),
+                                   pack_bf16(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv),
+                                   pack_bf16(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv),
+                                   pack_bf16(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv));
+            }
+        }
+    }
+    return true;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     packed_attention_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                             const __grid_constant__ CUtensorMap tm_vt, const AttnArgs a) {
@@ -256,23 +423,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t *base = dyn_smem + ((1024u - (saddr(dyn_smem) & 1023u)) & 1023u);
     uint8_t *sq = base;
-    uint8_t *skv = base + kQBytes;
-    uint8_t *sp = skv + kKvStages * kKvBytes;
+    uint8_t *sk = sq + kQBytes;                  // K stages
+    uint8_t *sv = sk + kKvStages * kKBytes;      // V^T stages
 
     if (threadIdx.x == 0) {
         mbar_init(&c.q_full, 1);
         mbar_init(&c.q_empty, 1);
         for (int s = 0; s < kKvStages; ++s) {
-            mbar_init(&c.kv_full[s], 1);
-            mbar_init(&c.kv_empty[s], 1);
+            mbar_init(&c.k_full[s], 1);
+            mbar_init(&c.k_empty[s], 1);
+            mbar_init(&c.v_full[s], 1);
+            mbar_init(&c.v_empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) mbar_init(&c.s_full[b], 1);
+        for (int b = 0; b < kPBufs; ++b) mbar_init(&c.pv_done[b], 1);
         mbar_init(&c.p_full, kSoftWarps);
-        mbar_init(&c.pv_done, 1);
-        mbar_init(&c.o_free, kSoftWarps);
+        for (int b = 0; b < 2; ++b) mbar_init(&c.o_free[b], kSoftWarps);
         mbar_init(&c.mma_done, 1);
         c.abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    for (int i = threadIdx.x; i < 2 * 2 * kBQ; i += kThreads) {  // stamp 0: nothing published
+        (&c.xmax[0][0][0])[i] = 0;
+        (&c.xsum[0][0][0])[i] = 0;
     }
     if (warp == 1) {
         tmem_alloc(&c.tmem_base, kTmemCols);
@@ -287,7 +460,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t idesc = umma::instr_desc_bf16(kBQ, kBK);
 
     if (warp == 0) {
-        if (lane == 0) {  // -------------------------------------------- TMA producer
+        if (lane == 0) {  // -------------------------------------------- Q and K producer
             uint32_t g = 0;  // key tiles issued (all items)
             int n_items = 0;
             bool ok = true;
@@ -300,79 +473,104 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tma_load_2d(sq + kAtom, &tm_q, 64, qrow, &c.q_full);
                 for (int j = 0; j < it.n_tiles; ++j, ++g) {
                     const int s = g % kKvStages;
-                    if (!wait_or_abort(&c.kv_empty[s], ((g / kKvStages) & 1) ^ 1, c, a)) {
+                    if (!wait_or_abort(&c.k_empty[s], ((g / kKvStages) & 1) ^ 1, c, a)) {
                         ok = false;
                         break;
                     }
                     int k0, valid;
                     key_tile(a, it, j, k0, valid);
-                    uint8_t *sk = skv + s * kKvBytes, *sv = sk + kKBytes;
-                    mbar_expect_tx(&c.kv_full[s], kKvBytes);
+                    uint8_t *dst = sk + s * kKBytes;
+                    mbar_expect_tx(&c.k_full[s], kKBytes);
                     const int krow = it.bh * a.n_tokens + k0;
-                    tma_load_2d(sk, &tm_k, 0, krow, &c.kv_full[s]);
-                    tma_load_2d(sk + kAtom, &tm_k, 64, krow, &c.kv_full[s]);
-                    tma_load_2d(sv, &tm_vt, k0, it.bh * kD, &c.kv_full[s]);
-                    tma_load_2d(sv + kAtom, &tm_vt, k0 + 64, it.bh * kD, &c.kv_full[s]);
+                    tma_load_2d(dst, &tm_k, 0, krow, &c.k_full[s]);
+                    tma_load_2d(dst + kAtom, &tm_k, 64, krow, &c.k_full[s]);
                 }
             }
             // every copy issued lands before the CTA leaves
             for (uint32_t j = g > kKvStages ? g - kKvStages : 0; j < g; ++j)
-                wait_drain(&c.kv_full[j % kKvStages], (j / kKvStages) & 1);
+                wait_drain(&c.k_full[j % kKvStages], (j / kKvStages) & 1);
             if (n_items > 0) wait_drain(&c.q_full, (n_items - 1) & 1);
+        }
+    } else if (warp == kVWarp) {
+        if (lane == 0) {  // -------------------------------------------- V producer
+            uint32_t g = 0;
+            bool ok = true;
+            for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x) {
+                const Item it = item_of(a, w);
+                for (int j = 0; j < it.n_tiles; ++j, ++g) {
+                    const int s = g % kKvStages;
+                    if (!wait_or_abort(&c.v_empty[s], ((g / kKvStages) & 1) ^ 1, c, a)) {
+                        ok = false;
+                        break;
+                    }
+                    int k0, valid;
+                    key_tile(a, it, j, k0, valid);
+                    uint8_t *dst = sv + s * kVBytes;
+                    mbar_expect_tx(&c.v_full[s], kVBytes);
+                    tma_load_2d(dst, &tm_vt, k0, it.bh * kD, &c.v_full[s]);
+                    tma_load_2d(dst + kAtom, &tm_vt, k0 + 64, it.bh * kD, &c.v_full[s]);
+                }
+            }
+            for (uint32_t j = g > kKvStages ? g - kKvStages : 0; j < g; ++j)
+                wait_drain(&c.v_full[j % kKvStages], (j / kKvStages) & 1);
         }
     } else if (warp == 1) {
         if (lane == 0) {  // -------------------------------------------- MMA issuer
             uint32_t g = 0;  // key tiles consumed (all items)
             int n_items = 0;
             bool ok = true;
+            const uint64_t qd = umma::smem_desc_kmajor_sw128(saddr(sq));
+            const uint64_t qd1 = umma::smem_desc_kmajor_sw128(saddr(sq + kAtom));
             for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x, ++n_items) {
                 const Item it = item_of(a, w);
                 if (!wait_or_abort(&c.q_full, n_items & 1, c, a)) break;
                 tc_fence_after();
-                const uint64_t qd = umma::smem_desc_kmajor_sw128(saddr(sq));
-                const uint64_t qd1 = umma::smem_desc_kmajor_sw128(saddr(sq + kAtom));
-                const uint64_t pd = umma::smem_desc_kmajor_sw128(saddr(sp));
-                const uint64_t pd1 = umma::smem_desc_kmajor_sw128(saddr(sp + kAtom));
                 for (int j = 0; j <= it.n_tiles && ok; ++j) {
                     if (j < it.n_tiles) {  // S_j = Q K_j^T
                         const uint32_t gj = g + j;
                         const int s = gj % kKvStages;
-                        if (!wait_or_abort(&c.kv_full[s], (gj / kKvStages) & 1, c, a)) {
+                        if (!wait_or_abort(&c.k_full[s], (gj / kKvStages) & 1, c, a)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        const uint8_t *sk = skv + s * kKvBytes;
-                        const uint64_t kd = umma::smem_desc_kmajor_sw128(saddr(sk));
-                        const uint64_t kd1 = umma::smem_desc_kmajor_sw128(saddr(sk + kAtom));
+                        const uint64_t kd = umma::smem_desc_kmajor_sw128(saddr(sk + s * kKBytes));
+                        const uint64_t kd1 = umma::smem_desc_kmajor_sw128(saddr(sk + s * kKBytes + kAtom));
                         const uint32_t sbuf = tmem + (gj & 1) * kBK;
 #pragma unroll
                         for (int k = 0; k < 8; ++k)
                             mma_bf16(sbuf, umma::advance_k16(k < 4 ? qd : qd1, k & 3),
                                      umma::advance_k16(k < 4 ? kd : kd1, k & 3), idesc, k != 0);
+                        mma_commit(&c.k_empty[s]);  // K stage free once S_j is computed
                         mma_commit(&c.s_full[gj & 1]);
                         if (j == it.n_tiles - 1) mma_commit(&c.q_empty);  // Q is no longer read
                     }
                     if (j >= 1) {  // O += P_{j-1} V_{j-1}
                         const uint32_t gp = g + j - 1;
-                        if (j == 1 && !wait_or_abort(&c.o_free, (n_items & 1) ^ 1, c, a)) {
+                        // O buffer n % 2 was last read out for item n - 2 (phase n / 2 - 1 of
+                        // its barrier; a fresh barrier passes parity 1 for items 0 and 1)
+                        if (j == 1 && !wait_or_abort(&c.o_free[n_items & 1], ((n_items >> 1) & 1) ^ 1, c, a)) {
                             ok = false;
                             break;
                         }
-                        if (!wait_or_abort(&c.p_full, gp & 1, c, a)) {
+                        if (!wait_or_abort(&c.p_full, gp & 1, c, a) ||
+                            !wait_or_abort(&c.v_full[gp % kKvStages], (gp / kKvStages) & 1, c, a)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        const uint8_t *sv = skv + (gp % kKvStages) * kKvBytes + kKBytes;
-                        const uint64_t vd = umma::smem_desc_kmajor_sw128(saddr(sv));
-                        const uint64_t vd1 = umma::smem_desc_kmajor_sw128(saddr(sv + kAtom));
+                        const uint8_t *vb = sv + (gp % kKvStages) * kVBytes;
+                        const uint64_t vd = umma::smem_desc_kmajor_sw128(saddr(vb));
+                        const uint64_t vd1 = umma::smem_desc_kmajor_sw128(saddr(vb + kAtom));
+                        // P of keys 16k..16k+15: columns (k / 4) * 64 + (k % 4) * 8 of S buffer gp % 2
+                        // (each half-row wrote its 64 keys, two per column, over its own first 32 columns)
+                        const uint32_t pcol = tmem + (gp & 1) * kBK;
 #pragma unroll
                         for (int k = 0; k < 8; ++k)
-                            mma_bf16(tmem + kOCol, umma::advance_k16(k < 4 ? pd : pd1, k & 3),
-                                     umma::advance_k16(k < 4 ? vd : vd1, k & 3), idesc, (j > 1 || k != 0) ? 1u : 0u);
-                        mma_commit(&c.kv_empty[gp % kKvStages]);
-                        mma_commit(&c.pv_done);
+                            mma_bf16_ts(tmem + kOCol + (n_items & 1) * kD, pcol + (k >> 2) * 64 + (k & 3) * 8,
+                                        umma::advance_k16(k < 4 ? vd : vd1, k & 3), idesc, (j > 1 || k != 0) ? 1u : 0u);
+                        mma_commit(&c.v_empty[gp % kKvStages]);
+                        mma_commit(&c.pv_done[gp & 1]);
                     }
                 }
                 g += it.n_tiles;
@@ -381,16 +579,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             wait_drain(&c.mma_done, 0);
         }
         __syncwarp();
-    } else {  // ---------------------------------------------------- softmax
-        const int q = warp & 3;
+    } else {  // ---------------------------------------------------- softmax (warps 2-9)
+        // warp w reads TMEM lane quarter w % 4 (rows 32 q .. 32 q + 31) and half
+        // h of each S row (keys 64 h .. 64 h + 63); the two halves of a row
+        // agree on its maximum through the exchange slots
+        const int q = warp & 3, h = (warp - 2) >> 2;
         const int r = q * 32 + lane;  // query row in the tile (TMEM lane)
         const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
         uint32_t g = 0;
+        uint32_t waited[kPBufs] = {0, 0};
+        // The read-out of item n is deferred until the first P of item n + 1 is
+        // out, so that it overlaps that item's first products (O is double-buffered).
+        Pending pend;
+        pend.active = false;
+        bool ok = true;
         int n_items = 0;
-        for (int w = blockIdx.x; w < a.items; w += gridDim.x, ++n_items) {
+        for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x, ++n_items) {
             const Item it = item_of(a, w);
+            const uint32_t ocol = kOCol + (n_items & 1) * kD;
             float m = -INFINITY, l = 0.f;
-            bool ok = true;
             for (int j = 0; j < it.n_tiles; ++j) {
                 const uint32_t gj = g + j;
                 if (!warp_wait_or_abort(&c.s_full[gj & 1], (gj >> 1) & 1, c, a)) {
@@ -400,17 +607,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 int k0, valid;
                 key_tile(a, it, j, k0, valid);
-                const uint32_t sbuf = tmem + lane_off + (gj & 1) * kBK;
-                // pass 1: the tile's largest visible score
-                float tmx = -INFINITY;
-                for (int ch = 0; ch < kBK / 32; ++ch) {
-                    float v[32];
-                    tmem_ld32(sbuf + ch * 32, v);
+                const uint32_t sbuf = tmem + lane_off + (gj & 1) * kBK + h * 64;
+                // this half-row's 64 scores in one round of loads
+                uint32_t sr[2][32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        if (ch * 32 + i < valid) tmx = fmaxf(tmx, v[i]);
+                for (int ch = 0; ch < 2; ++ch) tmem_ld32_async(sbuf + ch * 32, sr[ch]);
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch) tmem_wait_dep(sr[ch]);
+                if (valid < kBK) {  // keys past the segment's end take no weight
+#pragma unroll
+                    for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (h * 64 + ch * 32 + i >= valid) sr[ch][i] = __float_as_uint(-INFINITY);
                 }
-                const float tm = tmx * a.c;
+                // the half's largest score (eight independent chains), then the row's
+                float mx8[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(sr[ch][i]));
+                const float hmx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                        fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+                xput(&c.xmax[gj & 1][h][r], gj + 1, hmx);
+                float omx;
+                if (!xget(&c.xmax[gj & 1][h ^ 1][r], gj + 1, omx, c, a)) {
+                    ok = false;
+                    break;
+                }
+                const float tm = fmaxf(hmx, omx) * a.c;  // the same in both halves
                 float f = 1.f;
                 bool rescale = false;
                 if (m == -INFINITY) {
@@ -420,79 +647,68 @@ __global__ void __launch_bounds__(kThreads, 1)
                     m = tm;
                     rescale = true;
                 }
-                // P and O of the previous tile are free once its PV has completed
-                if (j >= 1) {
-                    if (!warp_wait_or_abort(&c.pv_done, (gj - 1) & 1, c, a)) {
+                // tcgen05.ld / st are warp-wide (.sync.aligned): the warp
+                // rescales its half of O together when any of its rows needs
+                // it, the other rows by f = 1. O must be quiet: the previous
+                // product done.
+                if (__any_sync(kFull, rescale)) {
+                    if (!wait_pv(gj - 1, waited, c, a)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    // tcgen05.ld / st are warp-wide (.sync.aligned): the warp
-                    // rescales together when any of its rows needs it, the
-                    // other rows by f = 1
-                    if (__any_sync(kFull, rescale)) {
-                        for (int ch = 0; ch < kD / 32; ++ch) {
-                            float o[32];
-                            tmem_ld32(tmem + lane_off + kOCol + ch * 32, o);
+                    for (int ch = 0; ch < 2; ++ch) {
+                        float o[32];
+                        tmem_ld32(tmem + lane_off + ocol + h * 64 + ch * 32, o);
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) o[i] *= f;
-                            tmem_st32(tmem + lane_off + kOCol + ch * 32, o);
-                        }
+                        for (int i = 0; i < 32; ++i) o[i] *= f;
+                        tmem_st32(tmem + lane_off + ocol + h * 64 + ch * 32, o);
                     }
                 }
                 l *= f;
-                // pass 2: P = 2^(s c - m) into the swizzled P tile (row r)
-                for (int ch = 0; ch < kBK / 32; ++ch) {
-                    float v[32];
-                    tmem_ld32(sbuf + ch * 32, v);
-                    uint32_t pk[16];
+                // P = 2^(s c - m) (a masked key gives 2^-inf = 0), bf16 pairs,
+                // over the first 32 columns of this half's S (already in registers)
+                const f2 cc = pack2(a.c, a.c), mm = pack2(-m, -m);
+                f2 lsum[4] = {pack2(0.f, 0.f), pack2(0.f, 0.f), pack2(0.f, 0.f), pack2(0.f, 0.f)};
+                uint32_t pk[32];
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch)
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {
-                        const float p0 = ch * 32 + i < valid ? ex2(fmaf(v[i], a.c, -m)) : 0.f;
-                        const float p1 = ch * 32 + i + 1 < valid ? ex2(fmaf(v[i + 1], a.c, -m)) : 0.f;
-                        l += p0 + p1;
-                        pk[i / 2] = pack_bf16(p0, p1);
+                        const f2 u = fma2(pack2(__uint_as_float(sr[ch][i]), __uint_as_float(sr[ch][i + 1])), cc, mm);
+                        float u0, u1;
+                        unpack2(u, u0, u1);
+                        const float p0 = ex2(u0), p1 = ex2(u1);
+                        lsum[(i >> 1) & 3] = add2(lsum[(i >> 1) & 3], pack2(p0, p1));
+                        pk[ch * 16 + i / 2] = pack_bf16(p0, p1);
                     }
-                    // 32 keys = four 16-byte chunks of one atom row
-                    const int atom = ch >> 1;
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int chunk = (ch & 1) * 4 + u;
-                        uint4 *dst = reinterpret_cast<uint4 *>(sp + atom * kAtom + r * 128 + ((chunk ^ (r & 7)) << 4));
-                        *dst = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-                    }
+                tmem_st32_u(sbuf, pk);
+                {
+                    float l0, l1;
+                    unpack2(add2(add2(lsum[0], lsum[1]), add2(lsum[2], lsum[3])), l0, l1);
+                    l += l0 + l1;
                 }
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // P visible to the MMA
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&c.p_full);
-            }
-            if (!ok) break;
-            const uint32_t glast = g + it.n_tiles - 1;
-            if (!warp_wait_or_abort(&c.pv_done, glast & 1, c, a)) break;
-            tc_fence_after();
-            // O / l of this row, bf16, to global memory
-            const bool live = r < it.q_len;
-            const float inv = 1.f / l;
-            __nv_bfloat16 *dst = a.out + (static_cast<int64_t>(it.bh) * a.n_tokens + it.q_start + r) * kD;
-            for (int ch = 0; ch < kD / 32; ++ch) {
-                float o[32];
-                tmem_ld32(tmem + lane_off + kOCol + ch * 32, o);
-                if (live) {
-                    uint4 *d4 = reinterpret_cast<uint4 *>(dst + ch * 32);
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        d4[u] = make_uint4(pack_bf16(o[8 * u] * inv, o[8 * u + 1] * inv),
-                                           pack_bf16(o[8 * u + 2] * inv, o[8 * u + 3] * inv),
-                                           pack_bf16(o[8 * u + 4] * inv, o[8 * u + 5] * inv),
-                                           pack_bf16(o[8 * u + 6] * inv, o[8 * u + 7] * inv));
+                if (j == 0 && pend.active) {
+                    if (!read_out(pend, waited, tmem, lane_off, r, h, lane, c, a)) {
+                        ok = false;
+                        break;
+                    }
+                    pend.active = false;
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&c.o_free);  // O may be overwritten by the next item
+            if (!ok) break;
+            pend.active = true;
+            pend.it = it;
+            pend.l = l;
+            pend.glast = g + it.n_tiles - 1;
+            pend.ocol = ocol;
+            pend.n = n_items;
             g += it.n_tiles;
         }
+        if (ok && pend.active) read_out(pend, waited, tmem, lane_off, r, h, lane, c, a);
     }
     tc_fence_before();
     __syncthreads();
