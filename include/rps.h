@@ -400,7 +400,25 @@ typedef struct {
     int32_t d;
     int64_t vocab;
     int64_t hidden_stride, unembed_stride;
+    int32_t unembed_packed; /* 0: unembed is [vocab][d] as above; 1: it was written by
+                               rps_lmhead_pack_unembed (unembed_stride is then unused) */
 } rps_lmhead;
+
+/*
+ * The unembedding in the LM head's packed tile layout (no counterpart in the
+ * paper; a one-time re-layout of a static weight). Each 256-token x 64-column
+ * block becomes one contiguous 32 KB image, so that the LM head reads the
+ * unembedding in whole blocks instead of 128 bytes from each of 256 rows; rows
+ * past the vocabulary are zero. rps_lmhead_packed_bytes gives the size (0 for
+ * invalid arguments: vocab out of range, d not a positive multiple of 64).
+ * unembed: [vocab][d] bf16, rows `stride` elements apart (a multiple of 8).
+ * One launch on `stream`; packed must not overlap unembed. Errors:
+ * RPS_ERR_INVALID_ARG for NULL or misaligned pointers, sizes out of range or a
+ * small output.
+ */
+size_t rps_lmhead_packed_bytes(int64_t vocab, int32_t d);
+rps_status rps_lmhead_pack_unembed(const void *unembed, int64_t vocab, int32_t d, int64_t stride, void *packed,
+                                   size_t packed_bytes, rps_stream_t stream);
 
 /* Workspace bytes of rps_lmhead_row_stats (k_max 0 for statistics only); 0 for
  * invalid arguments. The workspace needs no zeroing before its first use

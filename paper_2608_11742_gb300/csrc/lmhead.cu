@@ -79,6 +79,7 @@ struct __align__(16) LmPartial {
 
 struct LmArgs {
     int32_t n_rows, d, n_vt, splits, kmax, k;
+    const uint8_t *w_packed;  // unembedding in the packed tile layout, or nullptr (tensor map)
     int64_t vocab;
     LmPartial *part;   // [n_rows][splits]
     float2 *lists;     // [n_rows][splits][kmax]: (logit, token id as int bits)
@@ -125,6 +126,13 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
             saddr(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(saddr(bar))
         : "memory");
+}
+// Plain bulk copy of `bytes` contiguous bytes into shared memory, completing on `bar`.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     saddr(dst)),
+                 "l"(src), "r"(bytes), "r"(saddr(bar))
+                 : "memory");
 }
 __device__ __forceinline__ void prefetch_map(const CUtensorMap *map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -310,7 +318,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint8_t *sa = ring + s * kStageBytes;
                     mbar_expect_tx(&c.full[s], kStageBytes);
                     tma_load_2d(sa, &tm_h, kb * kTileK, rt * kTileM, &c.full[s]);
-                    tma_load_2d(sa + kABytes, &tm_w, kb * kTileK, vt * kTileN, &c.full[s]);
+                    if (a.w_packed)  // one contiguous 32 KB block, already in the swizzled image
+                        bulk_load(sa + kABytes, a.w_packed + (static_cast<int64_t>(vt) * kblocks + kb) * kBBytes,
+                                  kBBytes, &c.full[s]);
+                    else
+                        tma_load_2d(sa + kABytes, &tm_w, kb * kTileK, vt * kTileN, &c.full[s]);
                     ++it;
                 }
             }
@@ -416,20 +428,36 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int ch = 0; ch < kTileN / 32; ++ch) {
                 float v[32];
                 tmem_ld32(tbase + ch * 32, v);
-                float ps = 0.f, pt = 0.f;
+                const int nv = min(32, ncol - ch * 32);  // valid columns of this chunk (32 but in the last tile)
+                if (nv < 32) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (i >= nv) v[i] = -INFINITY;  // contributes 2^-inf = 0 and never enters the list
+                }
+                float ps[2] = {0.f, 0.f}, pt[2] = {0.f, 0.f};
+                uint32_t cand = 0;  // columns that pass the list's last entry
+                const float thr = KMAX > 0 ? st.lv[KMAX > 0 ? KMAX - 1 : 0] : INFINITY;
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                    const int cc = ch * 32 + i;
-                    if (cc < ncol) {
-                        const float u = fmaf(v[i], kLog2e, -st.B);
-                        const float e = ex2(u);
-                        ps += e;
-                        pt = fmaf(u, e, pt);
-                        if (KMAX > 0 && v[i] > st.lv[KMAX > 0 ? KMAX - 1 : 0]) list_insert<KMAX>(st, v[i], col0 + cc);
-                    }
+                    const float u = fmaf(v[i], kLog2e, -st.B);
+                    const float e = ex2(u);
+                    ps[i & 1] += e;
+                    pt[i & 1] = fmaf(e > 0.f ? u : 0.f, e, pt[i & 1]);
+                    if (KMAX > 0 && v[i] > thr) cand |= 1u << i;
                 }
-                st.s += ps;
-                st.t += pt;
+                st.s += ps[0] + ps[1];
+                st.t += pt[0] + pt[1];
+                // the few candidates, one copy of the insertion (the list only
+                // grows stricter, so each is checked again against it)
+#pragma unroll 1
+                while (KMAX > 0 && cand) {
+                    const int i = __ffs(cand) - 1;
+                    cand &= cand - 1;
+                    float x = v[0];
+#pragma unroll
+                    for (int j = 1; j < 32; ++j) x = j == i ? v[j] : x;
+                    if (x > st.lv[KMAX > 0 ? KMAX - 1 : 0]) list_insert<KMAX>(st, x, col0 + ch * 32 + i);
+                }
                 if (a.logits_out && live) {
                     float *dst = a.logits_out + static_cast<int64_t>(row) * a.vocab + col0 + ch * 32;
                     for (int i = 0; i < 32; ++i)
@@ -593,6 +621,29 @@ __global__ void __launch_bounds__(kMergeThreads) lmhead_merge_kernel(const LmArg
     }
 }
 
+// ---------------------------------------------------------------- packed unembedding
+// The packed layout holds, for vocabulary tile vt and d slice kb, the 256 x 64
+// block W[256 vt + n][64 kb + k] as the 32 KB image a TMA load with 128-byte
+// swizzle would leave in shared memory: row n at byte 128 n, its 16-byte
+// chunk c at chunk position c ^ (n % 8). Rows past the vocabulary are zero.
+// One thread per 16-byte chunk of the packed tensor.
+__global__ void pack_unembed_kernel(const uint4 *w, int64_t vocab, int32_t d, int64_t stride_elems, uint4 *out,
+                                    int64_t n_chunks) {
+    const int kblocks = d / kTileK;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_chunks;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t blk = i / (kBBytes / 16);
+        const int in = static_cast<int>(i - blk * (kBBytes / 16));  // chunk within the block image
+        const int n = in >> 3, pos = in & 7, c = pos ^ (n & 7);     // row, stored position, source chunk
+        const int64_t vt = blk / kblocks;
+        const int kb = static_cast<int>(blk - vt * kblocks);
+        const int64_t row = vt * kTileN + n;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (row < vocab) v = w[(row * stride_elems + static_cast<int64_t>(kb) * kTileK) / 8 + c];
+        out[i] = v;
+    }
+}
+
 // ---------------------------------------------------------------- host
 struct LmDevice {
     bool ready = false;
@@ -672,6 +723,24 @@ using namespace rps;
 
 extern "C" {
 
+size_t rps_lmhead_packed_bytes(int64_t vocab, int32_t d) {
+    if (vocab < 1 || vocab > INT32_MAX || d < kTileK || d % kTileK) return 0;
+    return static_cast<size_t>((vocab + kTileN - 1) / kTileN) * (d / kTileK) * kBBytes;
+}
+
+rps_status rps_lmhead_pack_unembed(const void *unembed, int64_t vocab, int32_t d, int64_t stride, void *packed,
+                                   size_t packed_bytes, rps_stream_t stream) {
+    if (!unembed || !packed || reinterpret_cast<uintptr_t>(unembed) % 16 || reinterpret_cast<uintptr_t>(packed) % 16)
+        return RPS_ERR_INVALID_ARG;
+    const size_t need = rps_lmhead_packed_bytes(vocab, d);
+    if (need == 0 || stride < d || stride % 8 || packed_bytes < need) return RPS_ERR_INVALID_ARG;
+    const int64_t n_chunks = static_cast<int64_t>(need / 16);
+    const int grid = static_cast<int>(std::min<int64_t>((n_chunks + 255) / 256, 152 * 16));
+    pack_unembed_kernel<<<grid, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint4 *>(unembed), vocab, d, stride, static_cast<uint4 *>(packed), n_chunks);
+    return cudaGetLastError() == cudaSuccess ? RPS_OK : RPS_ERR_CUDA;
+}
+
 size_t rps_lmhead_workspace_bytes(int32_t n_rows, int64_t vocab, int32_t k_max) {
     if (n_rows < 1 || vocab < 1 || vocab > INT32_MAX || k_max < 0 || k_max > RPS_MAX_K) return 0;
     return lm_layout(n_rows, vocab, k_max).total;
@@ -682,8 +751,8 @@ rps_status rps_lmhead_row_stats(const rps_lmhead *lm, const rps_params *prm, con
     if (!lm || !lm->hidden || !lm->unembed || !out) return RPS_ERR_INVALID_ARG;
     if (lm->n_rows < 1 || lm->vocab < 1 || lm->vocab > INT32_MAX || lm->d < kTileK || lm->d % kTileK != 0)
         return RPS_ERR_INVALID_ARG;
-    if (lm->hidden_stride < lm->d || lm->unembed_stride < lm->d || lm->hidden_stride % 8 || lm->unembed_stride % 8)
-        return RPS_ERR_INVALID_ARG;
+    if (lm->hidden_stride < lm->d || lm->hidden_stride % 8) return RPS_ERR_INVALID_ARG;
+    if (!lm->unembed_packed && (lm->unembed_stride < lm->d || lm->unembed_stride % 8)) return RPS_ERR_INVALID_ARG;
     if (reinterpret_cast<uintptr_t>(lm->hidden) % 16 || reinterpret_cast<uintptr_t>(lm->unembed) % 16)
         return RPS_ERR_INVALID_ARG;
     if (!out->zmax || !out->lse || !out->H || !out->pmax || !out->argmax) return RPS_ERR_INVALID_ARG;
@@ -707,7 +776,11 @@ rps_status rps_lmhead_row_stats(const rps_lmhead *lm, const rps_params *prm, con
     const int splits = std::max(1, std::min({dev.sm_count / n_rt, n_vt, kMaxSplits}));
     CUtensorMap tm_h, tm_w;
     if ((st = make_map(&tm_h, lm->hidden, lm->n_rows, lm->d, lm->hidden_stride, kTileM)) != RPS_OK) return st;
-    if ((st = make_map(&tm_w, lm->unembed, lm->vocab, lm->d, lm->unembed_stride, kTileN)) != RPS_OK) return st;
+    if (lm->unembed_packed) {  // the tensor map is not read; the hidden map stands in its slot
+        tm_w = tm_h;
+    } else if ((st = make_map(&tm_w, lm->unembed, lm->vocab, lm->d, lm->unembed_stride, kTileN)) != RPS_OK) {
+        return st;
+    }
 
     LmArgs a;
     std::memset(&a, 0, sizeof a);
@@ -723,6 +796,7 @@ rps_status rps_lmhead_row_stats(const rps_lmhead *lm, const rps_params *prm, con
     a.part = reinterpret_cast<LmPartial *>(ws + w.part);
     a.lists = reinterpret_cast<float2 *>(ws + w.lists);
     a.logits_out = d_logits_out;
+    a.w_packed = lm->unembed_packed ? static_cast<const uint8_t *>(lm->unembed) : nullptr;
     a.err = err;
     a.wait_ns = ring_wait_limit_ns();
     a.zmax = out->zmax;

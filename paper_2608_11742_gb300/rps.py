@@ -117,9 +117,13 @@ _lib.rps_version.restype = C.c_int32
 _lib.rps_version.argtypes = []
 class RpsLmhead(C.Structure):
     _fields_ = [("hidden", _p), ("unembed", _p), ("n_rows", C.c_int32), ("d", C.c_int32), ("vocab", C.c_int64),
-                ("hidden_stride", C.c_int64), ("unembed_stride", C.c_int64)]
+                ("hidden_stride", C.c_int64), ("unembed_stride", C.c_int64), ("unembed_packed", C.c_int32)]
 
 
+_lib.rps_lmhead_packed_bytes.restype = C.c_size_t
+_lib.rps_lmhead_packed_bytes.argtypes = [C.c_int64, C.c_int32]
+_lib.rps_lmhead_pack_unembed.restype = C.c_int
+_lib.rps_lmhead_pack_unembed.argtypes = [_p, C.c_int64, C.c_int32, C.c_int64, _p, C.c_size_t, _p]
 _lib.rps_lmhead_workspace_bytes.restype = C.c_size_t
 _lib.rps_lmhead_workspace_bytes.argtypes = [C.c_int32, C.c_int64, C.c_int32]
 _lib.rps_lmhead_row_stats.restype = C.c_int
@@ -403,17 +407,35 @@ def rps_lmhead_workspace_bytes(n_rows: int, vocab: int, k_max: int) -> int:
     return n
 
 
+def rps_lmhead_pack_unembed(unembed: torch.Tensor, stream=None) -> torch.Tensor:
+    """The unembedding ``[V][d]`` (bf16 CUDA tensor) in the LM head's packed tile
+    layout, as a new uint8 CUDA tensor (a one-time re-layout of the weight)."""
+    if unembed.dtype != torch.bfloat16 or unembed.dim() != 2 or unembed.stride(1) != 1:
+        raise ValueError("unembed must be a bf16 [V][d] tensor with d contiguous")
+    V, d = unembed.shape
+    n = _lib.rps_lmhead_packed_bytes(V, d)
+    if n == 0:
+        raise RPSError(RPS_ERR_INVALID_ARG, "rps_lmhead_packed_bytes")
+    packed = torch.empty(n, dtype=torch.uint8, device=unembed.device)
+    _check(_lib.rps_lmhead_pack_unembed(unembed.data_ptr(), V, d, unembed.stride(0), packed.data_ptr(), n,
+                                        _stream(stream)), "rps_lmhead_pack_unembed")
+    return packed
+
+
 def rps_lmhead_row_stats(hidden: torch.Tensor, unembed: torch.Tensor, prm, out: RowStatsBuf, ws: torch.Tensor,
-                         logits_out: Optional[torch.Tensor] = None, stream=None) -> None:
+                         logits_out: Optional[torch.Tensor] = None, stream=None,
+                         packed: Optional[torch.Tensor] = None) -> None:
     """Row statistics of ``hidden @ unembed.T`` (bf16 CUDA tensors ``[n][d]`` and
     ``[V][d]``) into ``out``; ``logits_out`` (fp32 ``[n][V]``, testing) also
-    receives the logits."""
+    receives the logits. With ``packed`` (from rps_lmhead_pack_unembed of the
+    same unembedding) the kernel reads the packed copy instead."""
     if hidden.dtype != torch.bfloat16 or unembed.dtype != torch.bfloat16:
         raise TypeError("hidden and unembed must be bf16")
     if hidden.dim() != 2 or unembed.dim() != 2 or hidden.stride(1) != 1 or unembed.stride(1) != 1:
         raise ValueError("hidden [n][d] and unembed [V][d] with d contiguous")
-    lm = RpsLmhead(hidden.data_ptr(), unembed.data_ptr(), hidden.shape[0], hidden.shape[1], unembed.shape[0],
-                   hidden.stride(0), unembed.stride(0))
+    src = unembed.data_ptr() if packed is None else packed.data_ptr()
+    lm = RpsLmhead(hidden.data_ptr(), src, hidden.shape[0], hidden.shape[1], unembed.shape[0],
+                   hidden.stride(0), unembed.stride(0), 0 if packed is None else 1)
     p = params(prm) if prm is not None else None
     st = out.c()
     _check(_lib.rps_lmhead_row_stats(C.byref(lm), None if p is None else C.byref(p), C.byref(st), _ptr(logits_out),

@@ -125,3 +125,27 @@ def test_lmhead_wait_timeout_is_reported_and_the_workspace_recovers():
     assert rps.rps_poll_device_status() == (rps.RPS_OK, 0)
     o = oracle_default().row_stats(lmhead_logits(h, w), k)
     assert_close(stats_np(good).H, o.H, "H after re-zeroing")
+
+
+@pytest.mark.parametrize("n,d,V,k", [(200, 128, 1000, 10), (300, 256, 126464, 16), (64, 64, 151936, 0)])
+def test_lmhead_packed_unembedding_gives_the_same_bits(n, d, V, k):
+    """The packed tile layout holds the same operands in the order the tensor
+    cores read them: every statistic is bit-identical to the row-major path's."""
+    h, w = synth.lmhead_inputs(14, n, V, d)
+    hd, wd = dev_bf16(h), dev_bf16(w)
+    packed = rps.rps_lmhead_pack_unembed(wd)
+    outs = []
+    for pk in (None, packed):
+        out = rps.RowStatsBuf.alloc(n, k, "cuda")
+        ws = torch.empty(rps.rps_lmhead_workspace_bytes(n, V, k), dtype=torch.uint8, device="cuda")
+        rps.rps_workspace_init(ws)
+        rps.rps_lmhead_row_stats(hd, wd, Prm(k) if k else None, out, ws, packed=pk)
+        assert rps.rps_poll_device_status() == (rps.RPS_OK, 0)
+        outs.append(out)
+    from dataclasses import fields
+    for f in fields(outs[0]):
+        a, b = getattr(outs[0], f.name), getattr(outs[1], f.name)
+        if a is None:
+            continue
+        assert torch.equal(a.nan_to_num(-7.0) if a.is_floating_point() else a,
+                           b.nan_to_num(-7.0) if b.is_floating_point() else b), f.name
