@@ -53,13 +53,16 @@ constexpr int kQBytes = 2 * kAtom;           // Q tile: two atoms along d
 constexpr int kKBytes = 2 * kAtom;           // K tile: two atoms along d
 constexpr int kVBytes = 2 * kAtom;           // V^T tile: two atoms along the keys
 constexpr int kKvStages = 2;
-constexpr int kPBufs = 2;                    // P of tile j lives in TMEM, in place of S buffer j % 2
-constexpr int kSmemBytes = kQBytes + kKvStages * (kKBytes + kVBytes) + 1024;
-constexpr int kThreads = 352;                // warp 0 and 10 TMA, warp 1 MMA, warps 2-9 softmax
+constexpr int kQBufs = 2;                    // the next item's Q loads while this item runs
+constexpr int kSBufs = 3;                    // S (and P, in place) of key tile g in TMEM buffer g % 3
+constexpr int kStageBytes = 32 * 64;           // per softmax warp: 32 rows x 32 bf16 of O on their way out
+constexpr int kSmemBytes = kQBufs * kQBytes + kKvStages * (kKBytes + kVBytes) + 8 * kStageBytes + 1024;
+constexpr int kThreads = 384;                // warps 0 and 10 TMA, 1 and 11 MMA, 2-9 softmax
 constexpr int kSoftWarps = 8;                // two per TMEM lane quarter: one per half of the keys
 constexpr int kVWarp = 10;
-constexpr uint32_t kTmemCols = 512;          // S buffers at columns 0 and 128, O buffers at 256 and 384
-constexpr uint32_t kOCol = 256;              // O of item n at kOCol + (n % 2) * kD
+constexpr int kPvWarp = 11;
+constexpr uint32_t kTmemCols = 512;          // S buffers at columns 0, 128 and 256, O at 384
+constexpr uint32_t kOCol = kSBufs * kBK;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescale = 8.0f;             // base-2 units a score may pass the reference by
 constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
@@ -149,6 +152,16 @@ __device__ __forceinline__ void tmem_st32_u(uint32_t taddr, const uint32_t (&v)[
         "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
         : "memory");
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr)
+                 : "memory");
+    return v;
 }
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(saddr(bar))
@@ -286,9 +299,22 @@ __device__ __forceinline__ void key_tile(const AttnArgs &a, const Item &it, int 
     }
 }
 
+// Moves (item n, key tile j) of the CTA's key-tile sequence one tile on:
+// the loops walk the sequence in order, with no division per tile.
+__device__ __forceinline__ void next_tile(int &n, int &j, int T) {
+    if (++j == T) {
+        j = 0;
+        ++n;
+    }
+}
+
 struct Ctl {
-    uint64_t q_full, q_empty, k_full[kKvStages], k_empty[kKvStages], v_full[kKvStages], v_empty[kKvStages];
-    uint64_t s_full[2], p_full, pv_done[kPBufs], o_free[2], mma_done;
+    uint64_t q_full[kQBufs], q_empty[kQBufs], k_full[kKvStages], k_empty[kKvStages], v_full[kKvStages],
+        v_empty[kKvStages];
+    // s_full and p_full per S / P buffer: the softmax may arrive on P up to three
+    // tiles ahead of the MMA's wait (P of tile u needs S of tile u, issued after
+    // the MMA saw P of tile u - 3), one phase ahead on each of three barriers
+    uint64_t s_full[kSBufs], p_full[kSBufs], pv_done[kSBufs], o_ready, o_free, mma_done;
     // the two halves of a row trade their tile maxima and, at the end of an
     // item, their sums: (stamp << 32 | value bits), double-buffered by parity
     uint64_t xmax[2][2][kBQ], xsum[2][2][kBQ];  // [parity][half][row]
@@ -323,17 +349,15 @@ __device__ void wait_drain(uint64_t *bar, uint32_t parity) {
         if (mbar_try_wait(bar, parity)) return;
 }
 
-// Waits (warp-wide) for the P V product of global key tile x, unless an
-// earlier wait already covered it. pv_done[x % 2] completes one phase per
-// product that reads P buffer x % 2; waited[b] counts the phases this thread
-// has seen, and a product is only waited for before the one two tiles later
-// can have been issued, so the parity names one phase.
-__device__ __forceinline__ bool wait_pv(uint32_t x, uint32_t (&waited)[kPBufs], Ctl &c, const AttnArgs &a) {
-    const uint32_t b = x & 1, ph = x >> 1;
-    if (waited[b] > ph) return true;
-    if (!warp_wait_or_abort(&c.pv_done[b], ph & 1, c, a)) return false;
-    waited[b] = ph + 1;
-    return true;
+// Waits (warp-wide) until the P V product of global key tile x has completed.
+// Product x completes phase x / 3 of pv_done[x % 3] (one phase per product
+// that reads P from S buffer x % 3). The softmax waits for it at tile x + 1,
+// before a rescale of O: S of tile x + 1 was issued only after product x - 2
+// had completed, and product x + 3 needs P that this softmax has not made, so
+// the barrier is at phase x / 3 (pending) or x / 3 + 1 (done), which its
+// parity tells apart.
+__device__ __forceinline__ bool wait_pv(uint32_t x, Ctl &c, const AttnArgs &a) {
+    return warp_wait_or_abort(&c.pv_done[x % kSBufs], (x / kSBufs) & 1, c, a);
 }
 
 // Publishes this half-row's value for the partner half (stamp != 0).
@@ -365,52 +389,56 @@ __device__ bool xget(uint64_t *slot, uint32_t stamp, float &v, Ctl &c, const Att
     return __all_sync(kFull, ok);
 }
 
-// An item whose O still waits to be written out.
-struct Pending {
-    bool active;
-    Item it;
-    float l;
-    uint32_t glast, ocol;
-    int n;
-};
-
-// O / l of this thread's half-row of a finished item (64 of the 128 columns),
-// bf16, to global memory; then the item's O buffer is released to the MMA
-// (o_free of its parity). The row sum is the two halves' sums added in a
-// fixed order.
-__device__ bool read_out(const Pending &pd, uint32_t (&waited)[kPBufs], uint32_t tmem, uint32_t lane_off, int r,
-                         int h, int lane, Ctl &c, const AttnArgs &a) {
-    if (!wait_pv(pd.glast, waited, c, a)) return false;
+// O / l of this thread's half-row of item n (64 of the 128 columns), bf16, to
+// global memory, once the item's last product is done (o_ready, one phase per
+// item); then O is released to the MMA (o_free). The row sum is the two
+// halves' sums added in a fixed order.
+__device__ bool read_out(const Item &it, int n, float l_half, uint32_t tmem, uint32_t lane_off, int r, int h, int lane,
+                         uint32_t stage, Ctl &c, const AttnArgs &a) {
+    if (!warp_wait_or_abort(&c.o_ready, n & 1, c, a)) return false;
     tc_fence_after();
-    const uint32_t stamp = static_cast<uint32_t>(pd.n) + 1u;
-    xput(&c.xsum[pd.n & 1][h][r], stamp, pd.l);
+    const uint32_t stamp = static_cast<uint32_t>(n) + 1u;
+    xput(&c.xsum[n & 1][h][r], stamp, l_half);
     float other;
-    if (!xget(&c.xsum[pd.n & 1][h ^ 1][r], stamp, other, c, a)) return false;
-    const float l = h == 0 ? pd.l + other : other + pd.l;
-    const bool live = r < pd.it.q_len;
+    if (!xget(&c.xsum[n & 1][h ^ 1][r], stamp, other, c, a)) return false;
+    const float l = h == 0 ? l_half + other : other + l_half;
     const float inv = 1.f / l;
-    __nv_bfloat16 *dst = a.out + (static_cast<int64_t>(pd.it.bh) * a.n_tokens + pd.it.q_start + r) * kD + h * 64;
     uint32_t o[2][32];
 #pragma unroll
-    for (int ch = 0; ch < 2; ++ch) tmem_ld32_async(tmem + lane_off + pd.ocol + h * 64 + ch * 32, o[ch]);
+    for (int ch = 0; ch < 2; ++ch) tmem_ld32_async(tmem + lane_off + kOCol + h * 64 + ch * 32, o[ch]);
 #pragma unroll
     for (int ch = 0; ch < 2; ++ch) tmem_wait_dep(o[ch]);
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&c.o_free[pd.n & 1]);  // the buffer may take item n + 2
-    if (live) {
+    if (lane == 0) mbar_arrive(&c.o_free);  // O may take the next item
+    // The warp's 32 rows go out through its shared-memory stage, 32 columns at
+    // a time: written a row per thread, read back so that each store
+    // instruction covers 64 contiguous bytes of 8 rows (a row per thread would
+    // touch 32 lines per instruction). The 16-byte chunk index is XORed with
+    // bits 1-2 of the row, so that neither the writes nor the reads put two
+    // threads of a quarter-warp in one bank group.
+    const int row0 = r - lane;  // first row of the warp's lane quarter
+    __nv_bfloat16 *dst = a.out + (static_cast<int64_t>(it.bh) * a.n_tokens + it.q_start + row0) * kD + h * 64;
 #pragma unroll
-        for (int ch = 0; ch < 2; ++ch) {
-            uint4 *d4 = reinterpret_cast<uint4 *>(dst + ch * 32);
+    for (int ch = 0; ch < 2; ++ch) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const uint32_t *x = o[ch] + 8 * u;
-                d4[u] = make_uint4(pack_bf16(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv),
-                                   pack_bf16(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv),
-                                   pack_bf16(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv),
-                                   pack_bf16(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv));
-            }
+        for (int u = 0; u < 4; ++u) {
+            const uint32_t *x = o[ch] + 8 * u;
+            st_shared_v4(stage + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4),
+                         make_uint4(pack_bf16(__uint_as_float(x[0]) * inv, __uint_as_float(x[1]) * inv),
+                                    pack_bf16(__uint_as_float(x[2]) * inv, __uint_as_float(x[3]) * inv),
+                                    pack_bf16(__uint_as_float(x[4]) * inv, __uint_as_float(x[5]) * inv),
+                                    pack_bf16(__uint_as_float(x[6]) * inv, __uint_as_float(x[7]) * inv)));
         }
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int rr = i * 8 + (lane >> 2), cc = lane & 3;
+            const uint4 v = ld_shared_v4(stage + rr * 64 + ((cc ^ ((rr >> 1) & 3)) << 4));
+            if (row0 + rr < it.q_len)
+                *reinterpret_cast<uint4 *>(dst + static_cast<int64_t>(rr) * kD + ch * 32 + cc * 8) = v;
+        }
+        __syncwarp();  // the stage is rewritten next
     }
     return true;
 }
@@ -422,24 +450,38 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ Ctl c;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t *base = dyn_smem + ((1024u - (saddr(dyn_smem) & 1023u)) & 1023u);
-    uint8_t *sq = base;
-    uint8_t *sk = sq + kQBytes;                  // K stages
+    uint8_t *sq = base;                          // Q buffers
+    uint8_t *sk = sq + kQBufs * kQBytes;         // K stages
     uint8_t *sv = sk + kKvStages * kKBytes;      // V^T stages
+    uint8_t *so = sv + kKvStages * kVBytes;      // output stages of the softmax warps
+    // Every item has the same number of key tiles (the context's and one
+    // branch's), so the CTA's key tiles are numbered globally: tile t is tile
+    // t % T of the CTA's item t / T.
+    const int T = a.q_tiles_ctx + a.q_tiles_branch;
+    const int my_items = blockIdx.x < static_cast<unsigned>(a.items)
+                             ? (a.items - 1 - static_cast<int>(blockIdx.x)) / static_cast<int>(gridDim.x) + 1
+                             : 0;
+    const uint32_t tiles = static_cast<uint32_t>(my_items) * T;
 
     if (threadIdx.x == 0) {
-        mbar_init(&c.q_full, 1);
-        mbar_init(&c.q_empty, 1);
+        for (int b = 0; b < kQBufs; ++b) {
+            mbar_init(&c.q_full[b], 1);
+            mbar_init(&c.q_empty[b], 1);
+        }
         for (int s = 0; s < kKvStages; ++s) {
             mbar_init(&c.k_full[s], 1);
             mbar_init(&c.k_empty[s], 1);
             mbar_init(&c.v_full[s], 1);
             mbar_init(&c.v_empty[s], 1);
         }
-        for (int b = 0; b < 2; ++b) mbar_init(&c.s_full[b], 1);
-        for (int b = 0; b < kPBufs; ++b) mbar_init(&c.pv_done[b], 1);
-        mbar_init(&c.p_full, kSoftWarps);
-        for (int b = 0; b < 2; ++b) mbar_init(&c.o_free[b], kSoftWarps);
-        mbar_init(&c.mma_done, 1);
+        for (int b = 0; b < kSBufs; ++b) {
+            mbar_init(&c.s_full[b], 1);
+            mbar_init(&c.p_full[b], kSoftWarps);
+        }
+        for (int b = 0; b < kSBufs; ++b) mbar_init(&c.pv_done[b], 1);
+        mbar_init(&c.o_ready, 1);
+        mbar_init(&c.o_free, kSoftWarps);
+        mbar_init(&c.mma_done, 2);  // one commit from each MMA issuer
         c.abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -461,119 +503,115 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 0) {
         if (lane == 0) {  // -------------------------------------------- Q and K producer
-            uint32_t g = 0;  // key tiles issued (all items)
-            int n_items = 0;
+            uint32_t t = 0;  // key tiles issued
+            int n_q = 0;     // Q tiles issued
             bool ok = true;
-            for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x, ++n_items) {
-                const Item it = item_of(a, w);
-                if (!wait_or_abort(&c.q_empty, (n_items & 1) ^ 1, c, a)) break;
-                mbar_expect_tx(&c.q_full, kQBytes);
-                const int qrow = it.bh * a.n_tokens + it.q_start;
-                tma_load_2d(sq, &tm_q, 0, qrow, &c.q_full);
-                tma_load_2d(sq + kAtom, &tm_q, 64, qrow, &c.q_full);
-                for (int j = 0; j < it.n_tiles; ++j, ++g) {
-                    const int s = g % kKvStages;
-                    if (!wait_or_abort(&c.k_empty[s], ((g / kKvStages) & 1) ^ 1, c, a)) {
-                        ok = false;
-                        break;
-                    }
-                    int k0, valid;
-                    key_tile(a, it, j, k0, valid);
-                    uint8_t *dst = sk + s * kKBytes;
-                    mbar_expect_tx(&c.k_full[s], kKBytes);
-                    const int krow = it.bh * a.n_tokens + k0;
-                    tma_load_2d(dst, &tm_k, 0, krow, &c.k_full[s]);
-                    tma_load_2d(dst + kAtom, &tm_k, 64, krow, &c.k_full[s]);
+            Item it{};
+            for (int n = 0, j = 0; t < tiles && ok; ++t, next_tile(n, j, T)) {
+                if (j == 0) {  // this item's Q, into buffer n % 2 once item n - 2 has left it
+                    it = item_of(a, blockIdx.x + n * gridDim.x);
+                    const int b = n & 1;
+                    if (!wait_or_abort(&c.q_empty[b], ((n >> 1) & 1) ^ 1, c, a)) break;
+                    mbar_expect_tx(&c.q_full[b], kQBytes);
+                    const int qrow = it.bh * a.n_tokens + it.q_start;
+                    tma_load_2d(sq + b * kQBytes, &tm_q, 0, qrow, &c.q_full[b]);
+                    tma_load_2d(sq + b * kQBytes + kAtom, &tm_q, 64, qrow, &c.q_full[b]);
+                    ++n_q;
                 }
+                const int s = t % kKvStages;
+                if (!wait_or_abort(&c.k_empty[s], ((t / kKvStages) & 1) ^ 1, c, a)) {
+                    ok = false;
+                    break;
+                }
+                int k0, valid;
+                key_tile(a, it, j, k0, valid);
+                uint8_t *dst = sk + s * kKBytes;
+                mbar_expect_tx(&c.k_full[s], kKBytes);
+                const int krow = it.bh * a.n_tokens + k0;
+                tma_load_2d(dst, &tm_k, 0, krow, &c.k_full[s]);
+                tma_load_2d(dst + kAtom, &tm_k, 64, krow, &c.k_full[s]);
             }
             // every copy issued lands before the CTA leaves
-            for (uint32_t j = g > kKvStages ? g - kKvStages : 0; j < g; ++j)
-                wait_drain(&c.k_full[j % kKvStages], (j / kKvStages) & 1);
-            if (n_items > 0) wait_drain(&c.q_full, (n_items - 1) & 1);
+            for (uint32_t x = t > kKvStages ? t - kKvStages : 0; x < t; ++x)
+                wait_drain(&c.k_full[x % kKvStages], (x / kKvStages) & 1);
+            for (int n = n_q > kQBufs ? n_q - kQBufs : 0; n < n_q; ++n) wait_drain(&c.q_full[n & 1], (n >> 1) & 1);
         }
     } else if (warp == kVWarp) {
         if (lane == 0) {  // -------------------------------------------- V producer
-            uint32_t g = 0;
-            bool ok = true;
-            for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x) {
-                const Item it = item_of(a, w);
-                for (int j = 0; j < it.n_tiles; ++j, ++g) {
-                    const int s = g % kKvStages;
-                    if (!wait_or_abort(&c.v_empty[s], ((g / kKvStages) & 1) ^ 1, c, a)) {
-                        ok = false;
-                        break;
-                    }
-                    int k0, valid;
-                    key_tile(a, it, j, k0, valid);
-                    uint8_t *dst = sv + s * kVBytes;
-                    mbar_expect_tx(&c.v_full[s], kVBytes);
-                    tma_load_2d(dst, &tm_vt, k0, it.bh * kD, &c.v_full[s]);
-                    tma_load_2d(dst + kAtom, &tm_vt, k0 + 64, it.bh * kD, &c.v_full[s]);
-                }
+            uint32_t t = 0;
+            Item it{};
+            for (int n = 0, j = 0; t < tiles; ++t, next_tile(n, j, T)) {
+                if (j == 0) it = item_of(a, blockIdx.x + n * gridDim.x);
+                const int s = t % kKvStages;
+                if (!wait_or_abort(&c.v_empty[s], ((t / kKvStages) & 1) ^ 1, c, a)) break;
+                int k0, valid;
+                key_tile(a, it, j, k0, valid);
+                uint8_t *dst = sv + s * kVBytes;
+                mbar_expect_tx(&c.v_full[s], kVBytes);
+                tma_load_2d(dst, &tm_vt, k0, it.bh * kD, &c.v_full[s]);
+                tma_load_2d(dst + kAtom, &tm_vt, k0 + 64, it.bh * kD, &c.v_full[s]);
             }
-            for (uint32_t j = g > kKvStages ? g - kKvStages : 0; j < g; ++j)
-                wait_drain(&c.v_full[j % kKvStages], (j / kKvStages) & 1);
+            for (uint32_t x = t > kKvStages ? t - kKvStages : 0; x < t; ++x)
+                wait_drain(&c.v_full[x % kKvStages], (x / kKvStages) & 1);
         }
     } else if (warp == 1) {
-        if (lane == 0) {  // -------------------------------------------- MMA issuer
-            uint32_t g = 0;  // key tiles consumed (all items)
-            int n_items = 0;
+        if (lane == 0) {  // -------------------------------------------- S issuer
             bool ok = true;
-            const uint64_t qd = umma::smem_desc_kmajor_sw128(saddr(sq));
-            const uint64_t qd1 = umma::smem_desc_kmajor_sw128(saddr(sq + kAtom));
-            for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x, ++n_items) {
-                const Item it = item_of(a, w);
-                if (!wait_or_abort(&c.q_full, n_items & 1, c, a)) break;
-                tc_fence_after();
-                for (int j = 0; j <= it.n_tiles && ok; ++j) {
-                    if (j < it.n_tiles) {  // S_j = Q K_j^T
-                        const uint32_t gj = g + j;
-                        const int s = gj % kKvStages;
-                        if (!wait_or_abort(&c.k_full[s], (gj / kKvStages) & 1, c, a)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        const uint64_t kd = umma::smem_desc_kmajor_sw128(saddr(sk + s * kKBytes));
-                        const uint64_t kd1 = umma::smem_desc_kmajor_sw128(saddr(sk + s * kKBytes + kAtom));
-                        const uint32_t sbuf = tmem + (gj & 1) * kBK;
-#pragma unroll
-                        for (int k = 0; k < 8; ++k)
-                            mma_bf16(sbuf, umma::advance_k16(k < 4 ? qd : qd1, k & 3),
-                                     umma::advance_k16(k < 4 ? kd : kd1, k & 3), idesc, k != 0);
-                        mma_commit(&c.k_empty[s]);  // K stage free once S_j is computed
-                        mma_commit(&c.s_full[gj & 1]);
-                        if (j == it.n_tiles - 1) mma_commit(&c.q_empty);  // Q is no longer read
-                    }
-                    if (j >= 1) {  // O += P_{j-1} V_{j-1}
-                        const uint32_t gp = g + j - 1;
-                        // O buffer n % 2 was last read out for item n - 2 (phase n / 2 - 1 of
-                        // its barrier; a fresh barrier passes parity 1 for items 0 and 1)
-                        if (j == 1 && !wait_or_abort(&c.o_free[n_items & 1], ((n_items >> 1) & 1) ^ 1, c, a)) {
-                            ok = false;
-                            break;
-                        }
-                        if (!wait_or_abort(&c.p_full, gp & 1, c, a) ||
-                            !wait_or_abort(&c.v_full[gp % kKvStages], (gp / kKvStages) & 1, c, a)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        const uint8_t *vb = sv + (gp % kKvStages) * kVBytes;
-                        const uint64_t vd = umma::smem_desc_kmajor_sw128(saddr(vb));
-                        const uint64_t vd1 = umma::smem_desc_kmajor_sw128(saddr(vb + kAtom));
-                        // P of keys 16k..16k+15: columns (k / 4) * 64 + (k % 4) * 8 of S buffer gp % 2
-                        // (each half-row wrote its 64 keys, two per column, over its own first 32 columns)
-                        const uint32_t pcol = tmem + (gp & 1) * kBK;
-#pragma unroll
-                        for (int k = 0; k < 8; ++k)
-                            mma_bf16_ts(tmem + kOCol + (n_items & 1) * kD, pcol + (k >> 2) * 64 + (k & 3) * 8,
-                                        umma::advance_k16(k < 4 ? vd : vd1, k & 3), idesc, (j > 1 || k != 0) ? 1u : 0u);
-                        mma_commit(&c.v_empty[gp % kKvStages]);
-                        mma_commit(&c.pv_done[gp & 1]);
-                    }
+            int n = 0, j = 0;
+            for (uint32_t t = 0; t < tiles && ok; ++t, next_tile(n, j, T)) {  // S_t = Q K_t^T into buffer t % 3
+                const int qb = n & 1, s = t % kKvStages;
+                // the buffer holds P of tile t - 3 until that product has completed
+                // (it comes from the other issuer: issue order does not protect it)
+                if ((j == 0 && !wait_or_abort(&c.q_full[qb], (n >> 1) & 1, c, a)) ||
+                    (t >= kSBufs && !wait_or_abort(&c.pv_done[t % kSBufs], ((t - kSBufs) / kSBufs) & 1, c, a)) ||
+                    !wait_or_abort(&c.k_full[s], (t / kKvStages) & 1, c, a)) {
+                    ok = false;
+                    break;
                 }
-                g += it.n_tiles;
+                tc_fence_after();
+                const uint64_t qd = umma::smem_desc_kmajor_sw128(saddr(sq + qb * kQBytes));
+                const uint64_t qd1 = umma::smem_desc_kmajor_sw128(saddr(sq + qb * kQBytes + kAtom));
+                const uint64_t kd = umma::smem_desc_kmajor_sw128(saddr(sk + s * kKBytes));
+                const uint64_t kd1 = umma::smem_desc_kmajor_sw128(saddr(sk + s * kKBytes + kAtom));
+                const uint32_t sbuf = tmem + (t % kSBufs) * kBK;
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(sbuf, umma::advance_k16(k < 4 ? qd : qd1, k & 3), umma::advance_k16(k < 4 ? kd : kd1, k & 3),
+                             idesc, k != 0);
+                mma_commit(&c.k_empty[s]);  // K stage free once S is computed
+                mma_commit(&c.s_full[t % kSBufs]);
+                if (j == T - 1) mma_commit(&c.q_empty[qb]);  // this Q is no longer read
+            }
+            mma_commit(&c.mma_done);
+            wait_drain(&c.mma_done, 0);
+        }
+        __syncwarp();
+    } else if (warp == kPvWarp) {
+        if (lane == 0) {  // -------------------------------------------- P V issuer
+            bool ok = true;
+            int n = 0, j = 0;
+            for (uint32_t t = 0; t < tiles && ok; ++t, next_tile(n, j, T)) {  // O += P_t V_t
+                // the first product of an item overwrites O: the previous item's read-out must be done
+                if ((j == 0 && !wait_or_abort(&c.o_free, (n & 1) ^ 1, c, a)) ||
+                    !wait_or_abort(&c.p_full[t % kSBufs], (t / kSBufs) & 1, c, a) ||
+                    !wait_or_abort(&c.v_full[t % kKvStages], (t / kKvStages) & 1, c, a)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint8_t *vb = sv + (t % kKvStages) * kVBytes;
+                const uint64_t vd = umma::smem_desc_kmajor_sw128(saddr(vb));
+                const uint64_t vd1 = umma::smem_desc_kmajor_sw128(saddr(vb + kAtom));
+                // P of keys 16k..16k+15: columns (k / 4) * 64 + (k % 4) * 8 of S buffer t % 3
+                // (each half-row wrote its 64 keys, two per column, over its own first 32 columns)
+                const uint32_t pcol = tmem + (t % kSBufs) * kBK;
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16_ts(tmem + kOCol, pcol + (k >> 2) * 64 + (k & 3) * 8,
+                                umma::advance_k16(k < 4 ? vd : vd1, k & 3), idesc, (j > 0 || k != 0) ? 1u : 0u);
+                mma_commit(&c.v_empty[t % kKvStages]);
+                mma_commit(&c.pv_done[t % kSBufs]);
+                if (j == T - 1) mma_commit(&c.o_ready);  // the item's O is complete
             }
             mma_commit(&c.mma_done);
             wait_drain(&c.mma_done, 0);
@@ -586,129 +624,127 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int q = warp & 3, h = (warp - 2) >> 2;
         const int r = q * 32 + lane;  // query row in the tile (TMEM lane)
         const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-        uint32_t g = 0;
-        uint32_t waited[kPBufs] = {0, 0};
-        // The read-out of item n is deferred until the first P of item n + 1 is
-        // out, so that it overlaps that item's first products (O is double-buffered).
-        Pending pend;
-        pend.active = false;
+        const uint32_t stage = saddr(so + (warp - 2) * kStageBytes);
+        float m = -INFINITY, l = 0.f;
+        // The read-out of item n waits until the first P of item n + 1 is out:
+        // by then its last product has had the softmax of a whole tile to finish.
+        Item pend_it{};
+        int pend_n = -1;
+        float pend_l = 0.f;
         bool ok = true;
-        int n_items = 0;
-        for (int w = blockIdx.x; w < a.items && ok; w += gridDim.x, ++n_items) {
-            const Item it = item_of(a, w);
-            const uint32_t ocol = kOCol + (n_items & 1) * kD;
-            float m = -INFINITY, l = 0.f;
-            for (int j = 0; j < it.n_tiles; ++j) {
-                const uint32_t gj = g + j;
-                if (!warp_wait_or_abort(&c.s_full[gj & 1], (gj >> 1) & 1, c, a)) {
+        Item it{};
+        int n = 0, j = 0;
+        for (uint32_t t = 0; t < tiles && ok; ++t, next_tile(n, j, T)) {
+            if (j == 0) {
+                it = item_of(a, blockIdx.x + n * gridDim.x);
+                m = -INFINITY;
+                l = 0.f;
+            }
+            const int sb = t % kSBufs;
+            if (!warp_wait_or_abort(&c.s_full[sb], (t / kSBufs) & 1, c, a)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            int k0, valid;
+            key_tile(a, it, j, k0, valid);
+            const uint32_t sbuf = tmem + lane_off + sb * kBK + h * 64;
+            // this half-row's 64 scores in one round of loads
+            uint32_t sr[2][32];
+#pragma unroll
+            for (int ch = 0; ch < 2; ++ch) tmem_ld32_async(sbuf + ch * 32, sr[ch]);
+#pragma unroll
+            for (int ch = 0; ch < 2; ++ch) tmem_wait_dep(sr[ch]);
+            if (valid < kBK) {  // keys past the segment's end take no weight
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (h * 64 + ch * 32 + i >= valid) sr[ch][i] = __float_as_uint(-INFINITY);
+            }
+            // the half's largest score (eight independent chains), then the row's
+            float mx8[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
+#pragma unroll
+            for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                for (int i = 0; i < 32; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(sr[ch][i]));
+            const float hmx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            xput(&c.xmax[t & 1][h][r], t + 1, hmx);
+            float omx;
+            if (!xget(&c.xmax[t & 1][h ^ 1][r], t + 1, omx, c, a)) {
+                ok = false;
+                break;
+            }
+            const float tm = fmaxf(hmx, omx) * a.c;  // the same in both halves
+            float f = 1.f;
+            bool rescale = false;
+            if (m == -INFINITY) {
+                m = tm;
+            } else if (tm > m + kRescale) {
+                f = ex2(m - tm);
+                m = tm;
+                rescale = true;
+            }
+            // tcgen05.ld / st are warp-wide (.sync.aligned): the warp rescales
+            // its half of O together when any of its rows needs it, the other
+            // rows by f = 1, once the product of the previous tile is done
+            if (__any_sync(kFull, rescale)) {
+                if (!wait_pv(t - 1, c, a)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                int k0, valid;
-                key_tile(a, it, j, k0, valid);
-                const uint32_t sbuf = tmem + lane_off + (gj & 1) * kBK + h * 64;
-                // this half-row's 64 scores in one round of loads
-                uint32_t sr[2][32];
+                for (int ch = 0; ch < 2; ++ch) {
+                    float o[32];
+                    tmem_ld32(tmem + lane_off + kOCol + h * 64 + ch * 32, o);
 #pragma unroll
-                for (int ch = 0; ch < 2; ++ch) tmem_ld32_async(sbuf + ch * 32, sr[ch]);
-#pragma unroll
-                for (int ch = 0; ch < 2; ++ch) tmem_wait_dep(sr[ch]);
-                if (valid < kBK) {  // keys past the segment's end take no weight
-#pragma unroll
-                    for (int ch = 0; ch < 2; ++ch)
-#pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (h * 64 + ch * 32 + i >= valid) sr[ch][i] = __float_as_uint(-INFINITY);
+                    for (int i = 0; i < 32; ++i) o[i] *= f;
+                    tmem_st32(tmem + lane_off + kOCol + h * 64 + ch * 32, o);
                 }
-                // the half's largest score (eight independent chains), then the row's
-                float mx8[8];
+            }
+            l *= f;
+            // P = 2^(s c - m) (a masked key gives 2^-inf = 0), bf16 pairs, over
+            // the first 32 columns of this half's S (already in registers)
+            const f2 cc = pack2(a.c, a.c), mm = pack2(-m, -m);
+            f2 lsum[4] = {pack2(0.f, 0.f), pack2(0.f, 0.f), pack2(0.f, 0.f), pack2(0.f, 0.f)};
+            uint32_t pk[32];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
+            for (int ch = 0; ch < 2; ++ch)
 #pragma unroll
-                for (int ch = 0; ch < 2; ++ch)
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(sr[ch][i]));
-                const float hmx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                        fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-                xput(&c.xmax[gj & 1][h][r], gj + 1, hmx);
-                float omx;
-                if (!xget(&c.xmax[gj & 1][h ^ 1][r], gj + 1, omx, c, a)) {
+                for (int i = 0; i < 32; i += 2) {
+                    const f2 u = fma2(pack2(__uint_as_float(sr[ch][i]), __uint_as_float(sr[ch][i + 1])), cc, mm);
+                    float u0, u1;
+                    unpack2(u, u0, u1);
+                    const float p0 = ex2(u0), p1 = ex2(u1);
+                    lsum[(i >> 1) & 3] = add2(lsum[(i >> 1) & 3], pack2(p0, p1));
+                    pk[ch * 16 + i / 2] = pack_bf16(p0, p1);
+                }
+            tmem_st32_u(sbuf, pk);
+            {
+                float l0, l1;
+                unpack2(add2(add2(lsum[0], lsum[1]), add2(lsum[2], lsum[3])), l0, l1);
+                l += l0 + l1;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&c.p_full[sb]);
+            if (j == 0 && pend_n >= 0) {
+                if (!read_out(pend_it, pend_n, pend_l, tmem, lane_off, r, h, lane, stage, c, a)) {
                     ok = false;
                     break;
                 }
-                const float tm = fmaxf(hmx, omx) * a.c;  // the same in both halves
-                float f = 1.f;
-                bool rescale = false;
-                if (m == -INFINITY) {
-                    m = tm;
-                } else if (tm > m + kRescale) {
-                    f = ex2(m - tm);
-                    m = tm;
-                    rescale = true;
-                }
-                // tcgen05.ld / st are warp-wide (.sync.aligned): the warp
-                // rescales its half of O together when any of its rows needs
-                // it, the other rows by f = 1. O must be quiet: the previous
-                // product done.
-                if (__any_sync(kFull, rescale)) {
-                    if (!wait_pv(gj - 1, waited, c, a)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    for (int ch = 0; ch < 2; ++ch) {
-                        float o[32];
-                        tmem_ld32(tmem + lane_off + ocol + h * 64 + ch * 32, o);
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) o[i] *= f;
-                        tmem_st32(tmem + lane_off + ocol + h * 64 + ch * 32, o);
-                    }
-                }
-                l *= f;
-                // P = 2^(s c - m) (a masked key gives 2^-inf = 0), bf16 pairs,
-                // over the first 32 columns of this half's S (already in registers)
-                const f2 cc = pack2(a.c, a.c), mm = pack2(-m, -m);
-                f2 lsum[4] = {pack2(0.f, 0.f), pack2(0.f, 0.f), pack2(0.f, 0.f), pack2(0.f, 0.f)};
-                uint32_t pk[32];
-#pragma unroll
-                for (int ch = 0; ch < 2; ++ch)
-#pragma unroll
-                    for (int i = 0; i < 32; i += 2) {
-                        const f2 u = fma2(pack2(__uint_as_float(sr[ch][i]), __uint_as_float(sr[ch][i + 1])), cc, mm);
-                        float u0, u1;
-                        unpack2(u, u0, u1);
-                        const float p0 = ex2(u0), p1 = ex2(u1);
-                        lsum[(i >> 1) & 3] = add2(lsum[(i >> 1) & 3], pack2(p0, p1));
-                        pk[ch * 16 + i / 2] = pack_bf16(p0, p1);
-                    }
-                tmem_st32_u(sbuf, pk);
-                {
-                    float l0, l1;
-                    unpack2(add2(add2(lsum[0], lsum[1]), add2(lsum[2], lsum[3])), l0, l1);
-                    l += l0 + l1;
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&c.p_full);
-                if (j == 0 && pend.active) {
-                    if (!read_out(pend, waited, tmem, lane_off, r, h, lane, c, a)) {
-                        ok = false;
-                        break;
-                    }
-                    pend.active = false;
-                }
+                pend_n = -1;
             }
-            if (!ok) break;
-            pend.active = true;
-            pend.it = it;
-            pend.l = l;
-            pend.glast = g + it.n_tiles - 1;
-            pend.ocol = ocol;
-            pend.n = n_items;
-            g += it.n_tiles;
+            if (j == T - 1) {
+                pend_it = it;
+                pend_n = n;
+                pend_l = l;
+            }
         }
-        if (ok && pend.active) read_out(pend, waited, tmem, lane_off, r, h, lane, c, a);
+        if (ok && pend_n >= 0) read_out(pend_it, pend_n, pend_l, tmem, lane_off, r, h, lane, stage, c, a);
     }
     tc_fence_before();
     __syncthreads();
