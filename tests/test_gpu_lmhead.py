@@ -89,10 +89,12 @@ def test_lmhead_parity(n, d, V, k):
     check(h, w, k)
 
 
-def test_lmhead_full_vocabulary_sampled_rows():
-    """300 rows x vocabulary 126,464: three row tiles, about ten vocabulary
-    tiles per CTA through both accumulators; twelve rows against the oracle."""
-    n, d, V, k = 300, 256, 126464, 10
+@pytest.mark.parametrize("n", [300, 256])
+def test_lmhead_full_vocabulary_sampled_rows(n):
+    """n rows x vocabulary 126,464, twelve rows against the oracle: three row
+    tiles (300 rows), or two (256 rows, the shape of a one-request step's base
+    rows), with several vocabulary tiles per CTA through both accumulators."""
+    d, V, k = 256, 126464, 10
     h, w = synth.lmhead_inputs(12, n, V, d)
     rows = np.random.default_rng(0).choice(n, 12, replace=False)
     check(h, w, k, rows)
