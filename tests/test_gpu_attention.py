@@ -61,6 +61,8 @@ def check(q, k, v, C, NB, G, scale):
     (2, 3, 200, 4, 40),    # ragged context and branches: the last key tile of each masks the rest
     (1, 2, 0, 3, 256),     # no context: each branch sees itself only
     (2, 4, 512, 9, 256),   # the lookahead shape: context 512, anchor + 8 branches of 256
+    (3, 8, 0, 9, 96),      # one key tile per item, several items per CTA: every tile ends an item
+    (4, 16, 64, 5, 64),    # two key tiles per item, two or three items per CTA
 ])
 def test_packed_attention_parity(n_b, n_h, C, NB, G):
     q, k, v = inputs(31, n_b, n_h, C, NB, G)
@@ -88,3 +90,19 @@ def test_packed_attention_isolation_bit_for_bit():
     keep[rows] = False
     assert np.array_equal(base[:, :, keep], moved[:, :, keep]), "another branch's output moved"
     assert not np.array_equal(base[:, :, rows], moved[:, :, rows])
+
+
+def test_packed_attention_full_size_sampled():
+    """The serving shape the bench times (8 requests x 32 heads, context 512,
+    anchor + 8 branches of 256: 2,816 packed tokens), one launch over all of it;
+    three (request, head) slices against the oracle."""
+    n_b, n_h, C, NB, G = 8, 32, 512, 9, 256
+    q, k, v = inputs(35, n_b, n_h, C, NB, G)
+    g = run_gpu(q, k, v, C, NB, G, 1.0 / np.sqrt(D))
+    for b, h in ((0, 0), (3, 17), (7, 31)):
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        ref = packed_attention(q[sl], k[sl], v[sl], C, NB, G, 1.0 / np.sqrt(D))
+        weighted_abs = packed_attention(q[sl], k[sl], v[sl] & np.uint16(0x7FFF), C, NB, G, 1.0 / np.sqrt(D))
+        tol = 2.0 ** -8 * (weighted_abs + np.abs(ref)) + 1e-6
+        err = np.abs(g[sl] - ref)
+        assert not (err > tol).any(), f"slice ({b}, {h}): {(err > tol).sum()} outputs out of tolerance"
