@@ -106,3 +106,22 @@ def test_packed_attention_full_size_sampled():
         tol = 2.0 ** -8 * (weighted_abs + np.abs(ref)) + 1e-6
         err = np.abs(g[sl] - ref)
         assert not (err > tol).any(), f"slice ({b}, {h}): {(err > tol).sum()} outputs out of tolerance"
+
+
+def test_packed_attention_wait_timeout_is_reported_and_the_next_launch_works():
+    """Every bounded wait gives up at once (testing hook): the launch reports
+    RPS_DEVERR_TIMEOUT and nothing hangs. Each role stops at its first wait, the
+    two MMA issuers drain, and TMEM is released: the next, normal launch
+    allocates it again and matches the oracle."""
+    C, NB, G = 256, 3, 128
+    q, k, v = inputs(36, 1, 2, C, NB, G)
+    out = torch.empty(q.shape, dtype=torch.bfloat16, device="cuda")
+    vt = np.ascontiguousarray(np.swapaxes(v, 2, 3))
+    rps.rps_debug_set_ring_wait_ns(0)
+    try:
+        rps.rps_packed_attention_fwd(dev(q), dev(k), dev(vt), out, C, NB, G, 0.1)
+        status, detail = rps.rps_poll_device_status()
+    finally:
+        rps.rps_debug_set_ring_wait_ns(2**64 - 1)
+    assert status == rps.RPS_ERR_DEVICE and detail & rps.DEVERR_TIMEOUT, hex(detail)
+    check(q, k, v, C, NB, G, 0.1)
