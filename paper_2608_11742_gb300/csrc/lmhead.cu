@@ -558,65 +558,67 @@ __global__ void __launch_bounds__(kMergeThreads) lmhead_merge_kernel(const LmArg
             a.argmax[row] = ok ? ram : -1;
             if (!ok) flag_error(a.err, RPS_DEVERR_NONFINITE);
         }
-        if (KMAX == 0 || a.k == 0) continue;
-        // k-way merge: rank r goes to lane r
-        for (int j = lane; j < a.splits; j += 32) head[j] = 0;
-        __syncwarp();
-        const float2 *ls = a.lists + static_cast<int64_t>(row) * a.splits * KMAX;
-        float tv = -INFINITY;
-        int ti = INT_MAX;
-        for (int r = 0; r < a.k; ++r) {
-            float bv = -INFINITY;
-            int bi = INT_MAX, bj = -1;
-#pragma unroll
-            for (int m = 0; m < kPerLane; ++m) {
-                const int j = lane + 32 * m;
-                if (j < a.splits && head[j] < KMAX) {
-                    const float2 e = ls[j * KMAX + head[j]];
-                    const int id = __float_as_int(e.y);
-                    if (bj < 0 || better(e.x, id, bv, bi)) {
-                        bv = e.x;
-                        bi = id;
-                        bj = j;
+        if constexpr (KMAX > 0) {  // (the statistics-only form has no lists)
+            if (a.k == 0) continue;
+            // k-way merge: rank r goes to lane r
+            for (int j = lane; j < a.splits; j += 32) head[j] = 0;
+            __syncwarp();
+            const float2 *ls = a.lists + static_cast<int64_t>(row) * a.splits * KMAX;
+            float tv = -INFINITY;
+            int ti = INT_MAX;
+            for (int r = 0; r < a.k; ++r) {
+                float bv = -INFINITY;
+                int bi = INT_MAX, bj = -1;
+    #pragma unroll
+                for (int m = 0; m < kPerLane; ++m) {
+                    const int j = lane + 32 * m;
+                    if (j < a.splits && head[j] < KMAX) {
+                        const float2 e = ls[j * KMAX + head[j]];
+                        const int id = __float_as_int(e.y);
+                        if (bj < 0 || better(e.x, id, bv, bi)) {
+                            bv = e.x;
+                            bi = id;
+                            bj = j;
+                        }
                     }
                 }
-            }
-            // warp-wide best (logit desc, token asc)
-            float wv = bv;
-            int wi = bi, wl = bj < 0 ? INT_MAX : lane;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const float ov = __shfl_xor_sync(kFull, wv, o);
-                const int oi = __shfl_xor_sync(kFull, wi, o);
-                const int ol = __shfl_xor_sync(kFull, wl, o);
-                if (ol != INT_MAX && (wl == INT_MAX || better(ov, oi, wv, wi))) {
-                    wv = ov;
-                    wi = oi;
-                    wl = ol;
+                // warp-wide best (logit desc, token asc)
+                float wv = bv;
+                int wi = bi, wl = bj < 0 ? INT_MAX : lane;
+    #pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const float ov = __shfl_xor_sync(kFull, wv, o);
+                    const int oi = __shfl_xor_sync(kFull, wi, o);
+                    const int ol = __shfl_xor_sync(kFull, wl, o);
+                    if (ol != INT_MAX && (wl == INT_MAX || better(ov, oi, wv, wi))) {
+                        wv = ov;
+                        wi = oi;
+                        wl = ol;
+                    }
                 }
+                if (lane == wl) ++head[bj];
+                if (lane == r) {
+                    tv = wl == INT_MAX ? -INFINITY : wv;
+                    ti = wl == INT_MAX ? INT_MAX : wi;
+                }
+                __syncwarp();
             }
-            if (lane == wl) ++head[bj];
-            if (lane == r) {
-                tv = wl == INT_MAX ? -INFINITY : wv;
-                ti = wl == INT_MAX ? INT_MAX : wi;
+            // mu and the truncated entropy against the row's reference, as the streaming kernel forms them
+            float p = 0.f, h = 0.f;
+            if (ok && lane < a.k && ti != INT_MAX) {
+                const float u = fmaf(tv, kLog2e, -M);
+                p = ex2(u) * invS;
+                if (p > 0.f) h = -p * (u * kLn2 - lnS);
             }
-            __syncwarp();
-        }
-        // mu and the truncated entropy against the row's reference, as the streaming kernel forms them
-        float p = 0.f, h = 0.f;
-        if (ok && lane < a.k && ti != INT_MAX) {
-            const float u = fmaf(tv, kLog2e, -M);
-            p = ex2(u) * invS;
-            if (p > 0.f) h = -p * (u * kLn2 - lnS);
-        }
-        const float mu = warp_sum(p), ht = warp_sum(h);
-        if (lane == 0) {
-            a.mu[row] = ok ? mu : NAN;
-            a.htrunc[row] = ok ? ht : NAN;
-        }
-        if (lane < a.k) {
-            a.topk_idx[static_cast<int64_t>(row) * a.k + lane] = ti == INT_MAX ? -1 : ti;
-            a.topk_logit[static_cast<int64_t>(row) * a.k + lane] = ti == INT_MAX ? NAN : tv;
+            const float mu = warp_sum(p), ht = warp_sum(h);
+            if (lane == 0) {
+                a.mu[row] = ok ? mu : NAN;
+                a.htrunc[row] = ok ? ht : NAN;
+            }
+            if (lane < a.k) {
+                a.topk_idx[static_cast<int64_t>(row) * a.k + lane] = ti == INT_MAX ? -1 : ti;
+                a.topk_logit[static_cast<int64_t>(row) * a.k + lane] = ti == INT_MAX ? NAN : tv;
+            }
         }
     }
 }
