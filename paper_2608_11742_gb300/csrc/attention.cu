@@ -265,18 +265,51 @@ struct Item {
     int n_ctx_tiles, n_tiles;   // key tiles: context tiles first
 };
 
-__device__ __forceinline__ Item item_of(const AttnArgs &a, int w) {
+// The CTA's items w = blockIdx.x + n * gridDim.x, walked in order: (bh, index
+// within bh) moves on by the grid's quotient and remainder, so the walk needs
+// no division per item (one at the start).
+struct ItemWalk {
+    int per_bh, step_bh, step_t;  // items per (batch, head); gridDim.x = step_bh * per_bh + step_t
+    int bh, t;                    // the current item
+    float inv_qtb;                // 1 / query tiles per branch
+};
+
+__device__ __forceinline__ ItemWalk item_walk(const AttnArgs &a) {
+    ItemWalk wk;
+    wk.per_bh = a.q_tiles_ctx + a.n_branch * a.q_tiles_branch;
+    wk.bh = static_cast<int>(blockIdx.x) / wk.per_bh;
+    wk.t = static_cast<int>(blockIdx.x) - wk.bh * wk.per_bh;
+    wk.step_bh = static_cast<int>(gridDim.x) / wk.per_bh;
+    wk.step_t = static_cast<int>(gridDim.x) - wk.step_bh * wk.per_bh;
+    wk.inv_qtb = 1.f / static_cast<float>(a.q_tiles_branch);
+    return wk;
+}
+
+__device__ __forceinline__ void item_next(ItemWalk &wk) {
+    wk.t += wk.step_t;
+    wk.bh += wk.step_bh;
+    if (wk.t >= wk.per_bh) {
+        wk.t -= wk.per_bh;
+        ++wk.bh;
+    }
+}
+
+// item_of for the walk's current item; the branch index is the float quotient
+// moved to the exact floor (it is off by at most one for these sizes; the
+// loops make the result exact regardless)
+__device__ __forceinline__ Item item_at(const AttnArgs &a, const ItemWalk &wk) {
     Item it;
-    const int per_bh = a.q_tiles_ctx + a.n_branch * a.q_tiles_branch;
-    it.bh = w / per_bh;
-    int t = w - it.bh * per_bh;
+    it.bh = wk.bh;
+    int t = wk.t;
     if (t < a.q_tiles_ctx) {
         it.seg_b = 0;
         it.q_start = t * kBQ;
         it.q_len = min(kBQ, a.n_context - it.q_start);
     } else {
         t -= a.q_tiles_ctx;
-        const int b = t / a.q_tiles_branch;
+        int b = __float2int_rz(static_cast<float>(t) * wk.inv_qtb);
+        while (b > 0 && b * a.q_tiles_branch > t) --b;
+        while ((b + 1) * a.q_tiles_branch <= t) ++b;
         const int qt = t - b * a.q_tiles_branch;
         it.seg_b = b;
         it.q_start = a.n_context + b * a.branch_len + qt * kBQ;
@@ -507,9 +540,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             int n_q = 0;     // Q tiles issued
             bool ok = true;
             Item it{};
+            ItemWalk wk = item_walk(a);
             for (int n = 0, j = 0; t < tiles && ok; ++t, next_tile(n, j, T)) {
                 if (j == 0) {  // this item's Q, into buffer n % 2 once item n - 2 has left it
-                    it = item_of(a, blockIdx.x + n * gridDim.x);
+                    if (n > 0) item_next(wk);
+                    it = item_at(a, wk);
                     const int b = n & 1;
                     if (!wait_or_abort(&c.q_empty[b], ((n >> 1) & 1) ^ 1, c, a)) break;
                     mbar_expect_tx(&c.q_full[b], kQBytes);
@@ -540,8 +575,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {  // -------------------------------------------- V producer
             uint32_t t = 0;
             Item it{};
+            ItemWalk wk = item_walk(a);
             for (int n = 0, j = 0; t < tiles; ++t, next_tile(n, j, T)) {
-                if (j == 0) it = item_of(a, blockIdx.x + n * gridDim.x);
+                if (j == 0) {
+                    if (n > 0) item_next(wk);
+                    it = item_at(a, wk);
+                }
                 const int s = t % kKvStages;
                 if (!wait_or_abort(&c.v_empty[s], ((t / kKvStages) & 1) ^ 1, c, a)) break;
                 int k0, valid;
@@ -633,10 +672,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         float pend_l = 0.f;
         bool ok = true;
         Item it{};
+        ItemWalk wk = item_walk(a);
         int n = 0, j = 0;
         for (uint32_t t = 0; t < tiles && ok; ++t, next_tile(n, j, T)) {
             if (j == 0) {
-                it = item_of(a, blockIdx.x + n * gridDim.x);
+                if (n > 0) item_next(wk);
+                it = item_at(a, wk);
                 m = -INFINITY;
                 l = 0.f;
             }
